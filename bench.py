@@ -1,0 +1,370 @@
+"""Benchmark of the RPD commit step on GB300.
+
+Default workload (N=1): the LLaDA-8B-shaped first step - batch 1, a 256-position canvas
+all masked, K=4 window layers, d=4096, V=126464 (1024 projected rows), tau 0.9, budget
+1.0 - with synthetic seeded inputs (the calibrated hidden-state recipe of ``workloads``).
+One "step" is one rpd_step call: gather + RMSNorm prologue, tcgen05 head statistics,
+split merge, scoring/scan/commit.  The canvas mask is restored before each step (a
+256-byte device copy) so every step sees the same workload.
+
+Metric: commit steps/s (and rows/s).  Under torchrun each rank runs its own canvas
+(weak scaling, no collective on the data path; a barrier and a max-reduce of the timer
+only).  ``--impl reference`` times the CPU oracle on a bounded sample of the same
+workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "RPD commit steps/s & rows/s at LLaDA-8B head shape; % of bf16 TC/HBM roofline"
+UNIT = "commit-steps/s"
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm_gbs=p["hbm_gbs"], bf16_tflops=p["bf16_tflops"],
+                    bf16_tflops_sustained=p.get("bf16_tflops_sustained", p["bf16_tflops"]),
+                    source="measured")
+    return dict(hbm_gbs=6800.0, bf16_tflops=1900.0, bf16_tflops_sustained=1700.0, source="fallback")
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock, power and throttle reasons, every 100 ms."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for _, ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def make_workload(rank: int):
+    import workloads as WL
+    W, g = WL.make_head(WL.LLADA_V, WL.LLADA_D, seed=2)
+    case = WL.llada_first_step(seed=2 + 97 * rank, W=W, g=g)
+    return case
+
+
+def rows_of(case):
+    return case["K"] * int(case["mask"].sum())
+
+
+def work_per_step(case):
+    """Algorithmic work of one step: FLOPs of the head contraction and the bytes of the
+    head (read once) plus the masked hidden rows."""
+    R = rows_of(case)
+    d, V = case["d"], case["V"]
+    flops = 2.0 * R * d * V
+    bytes_ = 2.0 * V * d + 2.0 * R * d
+    return R, flops, bytes_
+
+
+def cpu_oracle_rate(case, positions: int):
+    """Time the oracle (as it stands) on the first ``positions`` canvas positions of the
+    workload: returns (rows/s, seconds, threads)."""
+    from oracle import rpd_oracle as O
+    bits = lambda t: t.contiguous().view(torch.int16).numpy().view(np.uint16)  # noqa: E731
+    hb = bits(case["hidden"][:, :positions])
+    mask = np.ones(positions, dtype=np.uint8)
+    Wb, gb = bits(case["W"]), bits(case["g"])
+    t0 = time.perf_counter()
+    O.rpd_step(hb, mask, gb, Wb, case["eps"], case["tau"], case["budget"], case["rule"])
+    dt = time.perf_counter() - t0
+    threads = os.cpu_count() or 1
+    try:
+        from threadpoolctl import threadpool_info
+        blas = [i for i in threadpool_info() if i.get("user_api") == "blas"]
+        if blas:
+            threads = int(blas[0].get("num_threads", threads))
+    except Exception:
+        pass
+    return case["K"] * positions / dt, dt, threads
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    case = make_workload(0)
+    R, flops, bytes_ = work_per_step(case)
+    rates = []
+    # Each oracle call streams the whole head in fp64, so a call costs seconds: warm-up and
+    # timed calls stop once the run has used its time bound (at least one timed call).
+    t_start = time.perf_counter()
+    for _ in range(args.warmup):
+        cpu_oracle_rate(case, args.ref_positions)
+        if time.perf_counter() - t_start > args.ref_seconds / 4:
+            break
+    for _ in range(args.steps):
+        r, dt, threads = cpu_oracle_rate(case, args.ref_positions)
+        rates.append(r)
+        if time.perf_counter() - t_start > args.ref_seconds:
+            break
+    rows_s = statistics.median(rates)
+    steps_s = rows_s / R
+    out = {
+        "impl": "reference", "metric": METRIC, "value": steps_s, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / steps_s,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": config_dict(case, R),
+        "rows_per_s": rows_s,
+        "cpu_baseline": {"value": steps_s, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"{len(rates)} oracle calls (of {args.steps} requested, time bound "
+                                   f"{args.ref_seconds:.0f} s), each over the first {args.ref_positions} "
+                                   f"of 256 masked positions ({case['K'] * args.ref_positions} rows, "
+                                   f"full V and d); median rows/s scaled to the {R}-row step"},
+        "e2e": {"value": steps_s, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out))
+
+
+def config_dict(case, R):
+    return {"workload": "llada_first_step", "batch": 1, "N": case["N"], "K": case["K"],
+            "d": case["d"], "V": case["V"], "rows": R, "tau": case["tau"], "budget": case["budget"],
+            "rule": "llada (Table 4)", "signal_kappa": case.get("kappa"),
+            "l2": "inputs larger than L2: the 1.04 GB head is streamed every step"}
+
+
+def run_rpd(args):
+    rank, world, local = dist_env()
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    import paper_2609_36452_gb300 as rpd
+
+    case = make_workload(rank)
+    K, N, d, V = case["K"], case["N"], case["d"], case["V"]
+    R, flops, bytes_ = work_per_step(case)
+    W = case["W"].to(dev)
+    g = case["g"].to(dev)
+    hidden = case["hidden"].to(dev).contiguous()
+    mask0 = case["mask"].to(dev)
+    mask = mask0.clone()
+    commit = torch.zeros(N, dtype=torch.uint8, device=dev)
+    token = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    stats = torch.zeros(8, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    ctx = rpd.Rpd(d, V, K, case["eps"])
+    ctx.set_head(W, g)
+    ctx.set_profile(case["rule"])
+    ctx.set_stream(stream)
+    ctx.reserve(1, N)
+
+    def step():
+        mask.copy_(mask0, non_blocking=True)
+        ctx.step(hidden, mask, case["tau"], case["budget"], commit, token, stats)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    st = rpd.stats_dict(stats.cpu())
+    assert st["status"] == 0, st
+
+    ctx.kernel_times(reset=True)
+    ctx.profile(True)
+    barrier()
+    torch.cuda.synchronize(dev)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier()
+    ctx.profile(False)
+    clocks = sampler.stop() if sampler else None
+    ms_total = e0.elapsed_time(e1)
+    ktimes = ctx.kernel_times(reset=True)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms_total], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    steps_s = world * args.steps / (ms_total / 1e3)
+
+    # ---------------------------------------------------------------- end to end (host buffers)
+    hid_h = case["hidden"].contiguous().pin_memory()
+    mask_h0 = case["mask"].clone()
+    mask_h = mask_h0.clone().pin_memory()
+    commit_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
+    token_h = torch.full((N,), -1, dtype=torch.int32).pin_memory()
+    stats_h = torch.zeros(8, dtype=torch.int32).pin_memory()
+    e2e_steps = max(3, min(args.steps, 200))
+    for _ in range(2):
+        mask_h.copy_(mask_h0)
+        ctx.step_host(hid_h, mask_h, case["tau"], case["budget"], commit_h, token_h, stats_h)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        mask_h.copy_(mask_h0)
+        ctx.step_host(hid_h, mask_h, case["tau"], case["budget"], commit_h, token_h, stats_h)
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    h2d = hid_h.numel() * 2 + N + N * 4
+    d2h = N + N + N * 4 + 32
+
+    if rank != 0:
+        ctx.close()
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+
+    peaks = load_peaks()
+    head_ms, head_n = ktimes["head_stats"]
+    head_avg_ms = head_ms / max(head_n, 1)
+    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = bytes_ / (peaks["hbm_gbs"] * 1e9)
+    if t_tc >= t_hbm:
+        achieved = flops / (head_avg_ms * 1e-3) / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None,
+                "peak_kind": f"bf16 sustained, of {peaks['source']}",
+                "frac_of_burst": achieved / peaks["bf16_tflops"]}
+    else:
+        achieved = bytes_ / (head_avg_ms * 1e-3) / 1e9
+        peak = peaks["hbm_gbs"]
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": None, "peak_kind": f"HBM copy, of {peaks['source']}"}
+    step_roof = max(t_tc, t_hbm) / (ms_step * 1e-3)
+
+    cpu = None
+    if not args.no_cpu_baseline and world >= 1:
+        r_rows, dt, threads = cpu_oracle_rate(case, args.cpu_positions)
+        cpu = {"value": r_rows / R, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"oracle step over the first {args.cpu_positions} of 256 masked positions "
+                         f"({K * args.cpu_positions} rows, full V and d) took {dt:.1f} s; rows/s "
+                         f"scaled to the {R}-row step", "rows_per_s": r_rows}
+
+    out = {
+        "metric": METRIC, "value": steps_s, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": config_dict(case, R),
+        "rows_per_s": steps_s * R,
+        "roofline": roof,
+        "step_roofline_frac": step_roof,
+        "kernels_ms": {k: (v[0] / max(v[1], 1)) for k, v in ktimes.items()},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "api": "rpd_step_host (pinned host buffers)"},
+        "gpu_launches": 5 * args.steps,
+        "clocks": clocks,
+        "last_step_stats": st,
+    }
+    print(json.dumps(out))
+    ctx.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["rpd", "reference"], default="rpd")
+    ap.add_argument("--cpu-positions", type=int, default=32)
+    ap.add_argument("--ref-positions", type=int, default=8)
+    ap.add_argument("--ref-seconds", type=float, default=150.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_rpd(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,162 @@
+/*
+ * rpd.h - C ABI of the Reliable Parallel Decoding (RPD) commit step on one GPU.
+ *
+ * One call of rpd_step() performs one decoding iteration's commitment decision for a
+ * masked diffusion LM (paper §3): for every masked canvas position it projects the
+ * hidden states of the last K layers through the final RMSNorm and the LM head (the
+ * logit-lens readout of §2.2 and App. A.2, restricted to masked positions as App. A.6
+ * states), reads each layer's argmax and its probability and the final layer's
+ * confidence and entropy (Eq. 1), scores layerwise stability (Eq. 2-4), forms the
+ * candidate set (Eq. 5), and commits the candidates whose preceding masked positions
+ * hold at most `budget` nats of entropy (§3.2, E_i and A_t), falling back to the most
+ * confident of the first W masked positions when none qualifies (§3.2).
+ *
+ * Conventions for every entry point:
+ *  - Pointers named "device" are CUDA device pointers on the context's device; pointers
+ *    named "host" are host memory (pinned memory makes the copies asynchronous).
+ *  - bf16 arrays hold IEEE bfloat16 bit patterns (2 bytes per element).
+ *  - All device work is enqueued on the context's stream (rpd_set_stream) and is
+ *    asynchronous unless stated otherwise; nothing is read back to the host mid-step.
+ *  - Every int-returning function returns RPD_OK (0) or one of the RPD_ERR_* codes and
+ *    records a message for rpd_last_error() (per host thread).  On an error return no
+ *    output has been written unless the code is RPD_ERR_CUDA.
+ *  - A context is not thread safe; use one context per host thread or serialise calls.
+ */
+#ifndef RPD_H_
+#define RPD_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RPD_OK 0
+#define RPD_ERR_INVALID_ARGUMENT 1 /* bad size, pointer, threshold or alignment */
+#define RPD_ERR_NO_HEAD 2          /* rpd_step before rpd_set_head */
+#define RPD_ERR_CUDA 3             /* a CUDA runtime/driver call failed */
+#define RPD_ERR_OUT_OF_MEMORY 4    /* scratch allocation failed */
+#define RPD_ERR_TIMEOUT 5          /* a kernel's bounded wait ran out (latched in rpd_stats.status) */
+#define RPD_ERR_UNSUPPORTED 6      /* shape outside what the kernels handle */
+
+typedef struct rpd_ctx rpd_ctx; /* opaque, owned by the library */
+
+/* Rule parameters other than theta_h (= tau) and beta (= budget); Table 4 (App. A.6).
+ * rpd_create installs the LLaDA profile: theta_c 0.6, theta_s 3.5, w 15, k_max 6, window 32.
+ * The Dream profile is theta_s 2.5, w 20 with the rest unchanged. */
+typedef struct rpd_rule {
+    float theta_c;  /* minimum confidence for admission through stability (Eq. 5) */
+    float theta_s;  /* stability threshold (Eq. 5) */
+    float w;        /* weight of the confidence-drop penalty (Eq. 4), >= 0 */
+    int32_t k_max;  /* cap on prediction persistence (Eq. 4), >= 1 */
+    int32_t window; /* fallback window W: first W masked positions (§3.2), >= 1 */
+} rpd_rule;
+
+/* Per-canvas step summary, written to DEVICE memory by rpd_step / rpd_step_batched. */
+typedef struct rpd_stats {
+    int32_t n_masked;     /* |M_t| before the step */
+    int32_t n_candidates; /* |C_t| (Eq. 5) */
+    int32_t n_high_conf;  /* commits admitted through c >= theta_h */
+    int32_t n_stability;  /* commits admitted through theta_c <= c < theta_h and S >= theta_s */
+    int32_t n_committed;  /* positions committed this step, fallback included */
+    int32_t fallback_used;/* 1 if A_t was empty and the fallback commit was made */
+    int32_t fallback_pos; /* canvas index of the fallback commit, -1 if none */
+    int32_t status;       /* RPD_OK, or RPD_ERR_TIMEOUT if a kernel's bounded wait ran out */
+} rpd_stats;
+
+/* Optional per-position outputs (DEVICE pointers; any may be NULL).  Layouts use the
+ * step's B and N: "[B][N]" arrays are indexed b*N+i, "[K][B][N]" arrays (k*B+b)*N+i with
+ * k = 0 the earliest window layer and k = K-1 the final layer.  Unmasked positions get
+ * conf/entropy/drop/stability 0, persist 0, candidate 0, layer_argmax -1, layer_pmax 0. */
+typedef struct rpd_debug {
+    float *conf;          /* [B][N] c_i = p^(L)(y_i) */
+    float *entropy;       /* [B][N] H(p^(L)_i), nats */
+    int32_t *persist;     /* [B][N] K_i (Eq. 2) */
+    float *drop;          /* [B][N] r_i (Eq. 3) */
+    float *stability;     /* [B][N] S_i (Eq. 4) */
+    uint8_t *candidate;   /* [B][N] 1 if i in C_t */
+    int32_t *layer_argmax;/* [K][B][N] argmax token of each window layer */
+    float *layer_pmax;    /* [K][B][N] probability of that argmax */
+} rpd_debug;
+
+/* Create a context for hidden size d, vocabulary V, window K (the last K layers; the
+ * paper's l0 = L-K+1) and RMSNorm epsilon eps, on the current CUDA device.
+ * Requires d % 8 == 0 and d >= 64, V >= 256, 1 <= K <= 64, eps >= 0.
+ * Returns NULL on failure (see rpd_last_error()). */
+rpd_ctx *rpd_create(int d, int V, int K, float eps);
+
+/* Borrow the LM head W_head ([V][d] bf16, row v = token v's output embedding, device,
+ * 16-byte aligned) and the final-norm gain g_norm ([d] bf16, device, 16-byte aligned).
+ * Both must stay valid until the context is destroyed or the head is replaced; the
+ * library keeps no copy.  App. A.2: the model's own final normalisation and head. */
+int rpd_set_head(rpd_ctx *ctx, const void *W_head, const void *g_norm);
+
+/* Replace the rule parameters (Table 4).  Requires 0 <= theta_c, w >= 0, k_max >= 1,
+ * window >= 1.  theta_c < tau is checked per step (Eq. 5 requires theta_c < theta_h). */
+int rpd_set_rule(rpd_ctx *ctx, const rpd_rule *rule);
+int rpd_get_rule(const rpd_ctx *ctx, rpd_rule *rule);
+
+/* Run every later step on `stream` (a cudaStream_t; NULL = legacy default stream). */
+int rpd_set_stream(rpd_ctx *ctx, void *stream);
+
+/* Pre-size scratch for B canvases of N positions, so that later steps of that size
+ * allocate nothing.  Steps grow scratch on demand otherwise (synchronising the device). */
+int rpd_reserve(rpd_ctx *ctx, int B, int N);
+
+/* Install (or with NULL, clear) the optional per-position outputs. */
+int rpd_set_debug(rpd_ctx *ctx, const rpd_debug *debug);
+
+/* One commit step for one canvas (§3).
+ *   hidden     [K][N][d] bf16, device: pre-norm hidden state of each window layer at
+ *              each canvas position (the final layer last).  Rows of unmasked
+ *              positions are never read.
+ *   mask       [N] uint8, device, in/out: 1 = masked.  Committed positions are set to 0.
+ *   N          canvas length, 0 <= N <= 8192 (N = 0 is a no-op).
+ *   tau        theta_h, 0 < tau <= 1 and tau > theta_c.
+ *   budget     beta in nats, >= 0 (may be +inf).
+ *   out_commit [N] uint8, device: 1 where committed this step, 0 elsewhere.
+ *   out_token  [N] int32, device: y_i written ONLY at committed positions, so it may be
+ *              the canvas itself.
+ *   out_stats  one rpd_stats, device.
+ * With N_m > 0 masked positions at least one position is committed. */
+int rpd_step(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau, float budget,
+             uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats);
+
+/* B independent canvases of N positions in one step; the head is read once for all.
+ *   hidden [K][B][N][d] bf16 device; mask, out_commit, out_token [B][N] device;
+ *   tau, budget [B] HOST arrays (per-canvas theta_h and beta); out_stats [B] device.
+ * Requires 1 <= B <= 128. */
+int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int N,
+                     const float *tau, const float *budget, uint8_t *out_commit,
+                     int32_t *out_token, rpd_stats *out_stats);
+
+/* rpd_step with HOST buffers: copies hidden and mask in, runs the step, copies mask,
+ * out_commit, out_token and out_stats back, and returns after the stream has finished.
+ * Staging buffers are owned by the context (grown on demand).  mask is in/out. */
+int rpd_step_host(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau,
+                  float budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats);
+
+/* Per-kernel timing with CUDA events recorded on the context's stream around every
+ * launch while enabled.  rpd_kernel_times synchronises the recorded events and returns,
+ * for each of the RPD_NUM_KERNELS kernels (gather/norm, head statistics, merge,
+ * score/commit; the compaction kernel is counted with gather/norm), the summed
+ * milliseconds and the launch count since the last reset; reset clears them. */
+#define RPD_NUM_KERNELS 4
+int rpd_profile_enable(rpd_ctx *ctx, int enable);
+int rpd_kernel_times(rpd_ctx *ctx, double *ms /*[RPD_NUM_KERNELS]*/,
+                     int64_t *launches /*[RPD_NUM_KERNELS]*/, int reset);
+
+/* Free the context and its scratch (not the borrowed head).  NULL is ignored. */
+void rpd_destroy(rpd_ctx *ctx);
+
+/* Message of the last failing call on this host thread ("" if none). */
+const char *rpd_last_error(void);
+
+/* Library version string. */
+const char *rpd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RPD_H_ */

@@ -1,0 +1,223 @@
+"""RPD commit step on GB300 (sm_103a): Python binding of the C ABI in ``include/rpd.h``.
+
+The functions below carry the C names and only marshal arguments (ctypes); every step of
+the computation runs in the library's CUDA kernels.  PyTorch is used by callers for
+device memory and streams; the ``Rpd`` helper accepts torch tensors and passes their
+device pointers.  There is no CPU fallback: if ``librpd.so`` is missing or fails to
+load, importing the binding raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+__all__ = [
+    "RPD_OK", "RPD_ERR_INVALID_ARGUMENT", "RPD_ERR_NO_HEAD", "RPD_ERR_CUDA",
+    "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
+    "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
+    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_step",
+    "rpd_step_batched", "rpd_step_host", "rpd_profile_enable", "rpd_kernel_times",
+    "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
+]
+
+RPD_OK = 0
+RPD_ERR_INVALID_ARGUMENT = 1
+RPD_ERR_NO_HEAD = 2
+RPD_ERR_CUDA = 3
+RPD_ERR_OUT_OF_MEMORY = 4
+RPD_ERR_TIMEOUT = 5
+RPD_ERR_UNSUPPORTED = 6
+RPD_NUM_KERNELS = 4
+KERNEL_NAMES = ("gather_norm", "head_stats", "merge", "score_commit")
+
+# Table 4 (App. A.6) rule profiles: theta_c, theta_s, w, k_max, window.
+RULE_PROFILES = {
+    "llada": (0.6, 3.5, 15.0, 6, 32),
+    "dream": (0.6, 2.5, 20.0, 6, 32),
+}
+
+lib_path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librpd.so")
+
+
+class RpdRule(ctypes.Structure):
+    _fields_ = [("theta_c", ctypes.c_float), ("theta_s", ctypes.c_float), ("w", ctypes.c_float),
+                ("k_max", ctypes.c_int32), ("window", ctypes.c_int32)]
+
+
+class RpdStats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "n_masked", "n_candidates", "n_high_conf", "n_stability", "n_committed",
+        "fallback_used", "fallback_pos", "status")]
+
+
+class RpdDebug(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in (
+        "conf", "entropy", "persist", "drop", "stability", "candidate", "layer_argmax",
+        "layer_pmax")]
+
+
+STATS_FIELDS = [f[0] for f in RpdStats._fields_]
+
+
+class RpdError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"rpd error {code}: {msg}")
+        self.code = code
+
+
+def _load():
+    if not os.path.exists(lib_path):
+        raise ImportError(
+            f"{lib_path} is missing: build it with `python -c \"import __graft_entry__ as g; "
+            f"g.build()\"` (nvcc, sm_103a)")
+    L = ctypes.CDLL(lib_path)
+    vp, i32, f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    sig = {
+        "rpd_create": (vp, [i32, i32, i32, f32]),
+        "rpd_set_head": (i32, [vp, vp, vp]),
+        "rpd_set_rule": (i32, [vp, ctypes.POINTER(RpdRule)]),
+        "rpd_get_rule": (i32, [vp, ctypes.POINTER(RpdRule)]),
+        "rpd_set_stream": (i32, [vp, vp]),
+        "rpd_reserve": (i32, [vp, i32, i32]),
+        "rpd_set_debug": (i32, [vp, ctypes.POINTER(RpdDebug)]),
+        "rpd_step": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
+        "rpd_step_batched": (i32, [vp, vp, vp, i32, i32, vp, vp, vp, vp, vp]),
+        "rpd_step_host": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
+        "rpd_profile_enable": (i32, [vp, i32]),
+        "rpd_kernel_times": (i32, [vp, ctypes.POINTER(ctypes.c_double),
+                                   ctypes.POINTER(ctypes.c_int64), i32]),
+        "rpd_destroy": (None, [vp]),
+        "rpd_last_error": (ctypes.c_char_p, []),
+        "rpd_version": (ctypes.c_char_p, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    return L
+
+
+lib = _load()
+
+rpd_create = lib.rpd_create
+rpd_set_head = lib.rpd_set_head
+rpd_set_rule = lib.rpd_set_rule
+rpd_get_rule = lib.rpd_get_rule
+rpd_set_stream = lib.rpd_set_stream
+rpd_reserve = lib.rpd_reserve
+rpd_set_debug = lib.rpd_set_debug
+rpd_step = lib.rpd_step
+rpd_step_batched = lib.rpd_step_batched
+rpd_step_host = lib.rpd_step_host
+rpd_profile_enable = lib.rpd_profile_enable
+rpd_kernel_times = lib.rpd_kernel_times
+rpd_destroy = lib.rpd_destroy
+rpd_last_error = lib.rpd_last_error
+rpd_version = lib.rpd_version
+
+
+def _check(code: int):
+    if code != RPD_OK:
+        raise RpdError(code, rpd_last_error().decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+class Rpd:
+    """A context bound to torch tensors.  ``W`` ([V][d]) and ``g`` ([d]) are bf16 CUDA
+    tensors that must outlive the context (the library borrows them)."""
+
+    def __init__(self, d: int, V: int, K: int, eps: float = 1e-6):
+        self.d, self.V, self.K, self.eps = d, V, K, eps
+        h = rpd_create(d, V, K, ctypes.c_float(eps))
+        if not h:
+            raise RpdError(RPD_ERR_INVALID_ARGUMENT, rpd_last_error().decode())
+        self.handle = ctypes.c_void_p(h)
+        self._keep = []
+
+    def close(self):
+        if getattr(self, "handle", None):
+            rpd_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def set_head(self, W, g):
+        assert W.is_cuda and g.is_cuda and W.is_contiguous() and g.is_contiguous()
+        self._keep = [W, g]
+        _check(rpd_set_head(self.handle, _ptr(W), _ptr(g)))
+
+    def set_rule(self, theta_c, theta_s, w, k_max, window):
+        _check(rpd_set_rule(self.handle, ctypes.byref(RpdRule(theta_c, theta_s, w, k_max, window))))
+
+    def set_profile(self, name: str):
+        self.set_rule(*RULE_PROFILES[name])
+
+    def get_rule(self) -> dict:
+        r = RpdRule()
+        _check(rpd_get_rule(self.handle, ctypes.byref(r)))
+        return dict(theta_c=r.theta_c, theta_s=r.theta_s, w=r.w, k_max=r.k_max, window=r.window)
+
+    def set_stream(self, stream):
+        """``stream``: a torch.cuda.Stream, a raw cudaStream_t int, or None (legacy)."""
+        raw = getattr(stream, "cuda_stream", stream)
+        _check(rpd_set_stream(self.handle, ctypes.c_void_p(raw) if raw else None))
+
+    def reserve(self, B: int, N: int):
+        _check(rpd_reserve(self.handle, B, N))
+
+    def set_debug(self, **tensors):
+        """Keyword tensors named like the rpd_debug fields (CUDA, contiguous); None clears."""
+        if not tensors:
+            _check(rpd_set_debug(self.handle, None))
+            return
+        dbg = RpdDebug(*[_ptr(tensors.get(f)) if tensors.get(f) is not None else None
+                         for f, _ in RpdDebug._fields_])
+        self._dbg_keep = tensors
+        _check(rpd_set_debug(self.handle, ctypes.byref(dbg)))
+
+    def step(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
+        """One canvas: hidden [K][N][d] bf16, mask [N] uint8 (in/out), out_commit [N] uint8,
+        out_token [N] int32, out_stats int32 tensor of 8 (an rpd_stats), all CUDA."""
+        N = mask.numel()
+        _check(rpd_step(self.handle, _ptr(hidden), _ptr(mask), N, ctypes.c_float(tau),
+                        ctypes.c_float(budget), _ptr(out_commit), _ptr(out_token),
+                        _ptr(out_stats)))
+
+    def step_batched(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
+        """B canvases: hidden [K][B][N][d], mask/out_commit/out_token [B][N], out_stats [B][8];
+        tau and budget are length-B host sequences."""
+        B, N = mask.shape
+        ta = (ctypes.c_float * B)(*[float(x) for x in tau])
+        bu = (ctypes.c_float * B)(*[float(x) for x in budget])
+        _check(rpd_step_batched(self.handle, _ptr(hidden), _ptr(mask), B, N,
+                                ctypes.cast(ta, ctypes.c_void_p), ctypes.cast(bu, ctypes.c_void_p),
+                                _ptr(out_commit), _ptr(out_token), _ptr(out_stats)))
+
+    def step_host(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
+        """Host (CPU, ideally pinned) tensors; returns after the results are back."""
+        N = mask.numel()
+        _check(rpd_step_host(self.handle, _ptr(hidden), _ptr(mask), N, ctypes.c_float(tau),
+                             ctypes.c_float(budget), _ptr(out_commit), _ptr(out_token),
+                             _ptr(out_stats)))
+
+    def profile(self, enable: bool):
+        _check(rpd_profile_enable(self.handle, 1 if enable else 0))
+
+    def kernel_times(self, reset: bool = True):
+        ms = (ctypes.c_double * RPD_NUM_KERNELS)()
+        n = (ctypes.c_int64 * RPD_NUM_KERNELS)()
+        _check(rpd_kernel_times(self.handle, ms, n, 1 if reset else 0))
+        return {KERNEL_NAMES[i]: (ms[i], n[i]) for i in range(RPD_NUM_KERNELS)}
+
+
+def stats_dict(t) -> dict:
+    """Decode one rpd_stats (an int32 tensor/array of 8) into a dict."""
+    vals = [int(x) for x in (t.tolist() if hasattr(t, "tolist") else t)]
+    return dict(zip(STATS_FIELDS, vals))

@@ -1,0 +1,291 @@
+// k_merge_commit.cu - cross-split merge of the online softmax statistics, then the
+// scoring, candidate flags, entropy prefix scan and commitment of §3.
+//
+// k_merge (one warp per projected row): combines the row's G partials (m, s, t, a) in
+//   log2 units into the row's argmax a, its probability 1/s and the entropy
+//   H = ln s - ln2 * t / s  (Eq. 1; p_v = 2^(x_v - m) / s).
+//   Merge rule for partials j: m = max m_j, alpha_j = 2^(m_j - m),
+//   s = sum alpha_j s_j, t = sum alpha_j (t_j + (m_j - m) s_j); argmax = lowest index among
+//   the partials attaining m.
+//
+// k_score_commit (one CTA per canvas, positions in blocked order across threads):
+//   y_i = argmax of the final layer, c_i its probability, H_i its entropy;
+//   K_i = window layers, counted back from the final one, whose argmax is y_i (Eq. 2,
+//         stopping at the first disagreement, App. A.2);
+//   r_i = max over those layers of p(y_i) - c_i (Eq. 3; inside the suffix the layer argmax
+//         is y_i, so p(y_i) is that layer's maximum probability);
+//   S_i = min(K_i, K_max) - w r_i (Eq. 4);  cand_i per Eq. 5;
+//   Q_i = sum over j < i of H_j for masked non-candidates (block-wide exclusive scan);
+//   accept the candidates before the first candidate with Q > beta.  This equals the
+//   sequential rule of §3.2: H >= 0, accepted candidates are excluded from E_i, so while
+//   every earlier candidate was accepted E_i = Q_i, and after the first rejection every
+//   later candidate sees at least that much entropy.
+//   If nothing is accepted and something is masked, commit the most confident of the
+//   first W masked positions (leftmost on ties, §3.2).  Then write the outputs, clear the
+//   committed mask bits and the per-canvas counters.
+#include "rpd_internal.h"
+
+namespace rpd {
+namespace {
+
+constexpr float kLn2 = 0.6931471805599453f;
+
+struct Stat {
+    float m, s, t;
+    int a;
+};
+
+__device__ __forceinline__ Stat merge2(const Stat &x, const Stat &y) {
+    if (y.s <= 0.f) return x;
+    if (x.s <= 0.f) return y;
+    Stat r;
+    r.m = fmaxf(x.m, y.m);
+    const float dx = x.m - r.m, dy = y.m - r.m;
+    const float ax = exp2f(dx), ay = exp2f(dy);
+    r.s = ax * x.s + ay * y.s;
+    r.t = ax * fmaf(dx, x.s, x.t) + ay * fmaf(dy, y.s, y.t);
+    r.a = (x.m > y.m) ? x.a : (y.m > x.m) ? y.a : min(x.a, y.a);
+    return r;
+}
+
+__global__ void __launch_bounds__(256) k_merge(MergeParams p) {
+    const int rows = p.meta[kMetaRows];
+    const int splits = p.meta[kMetaSplits];
+    const int lane = threadIdx.x & 31;
+    const int wpc = blockDim.x >> 5;
+    for (int r = blockIdx.x * wpc + (threadIdx.x >> 5); r < rows; r += gridDim.x * wpc) {
+        Stat acc{-INFINITY, 0.f, 0.f, 0x7fffffff};
+        const float4 *row = p.partials + static_cast<size_t>(r) * p.max_splits;
+        for (int g = lane; g < splits; g += 32) {
+            const float4 v = row[g];
+            acc = merge2(acc, Stat{v.x, v.y, v.z, __float_as_int(v.w)});
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            Stat other;
+            other.m = __shfl_xor_sync(0xffffffffu, acc.m, o);
+            other.s = __shfl_xor_sync(0xffffffffu, acc.s, o);
+            other.t = __shfl_xor_sync(0xffffffffu, acc.t, o);
+            other.a = __shfl_xor_sync(0xffffffffu, acc.a, o);
+            // combine in lane order so every lane ends with the same bits
+            acc = (lane & o) ? merge2(other, acc) : merge2(acc, other);
+        }
+        if (lane == 0) {
+            p.row_arg[r] = acc.a;
+            p.row_pmax[r] = 1.0f / acc.s;
+            p.row_H[r] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ block-wide helpers
+
+template <typename T>
+__device__ __forceinline__ T warp_incl_scan(T v, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const T t = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += t;
+    }
+    return v;
+}
+
+// Exclusive scan over the block in thread order; `sh` holds 32 entries.
+template <typename T>
+__device__ __forceinline__ T block_excl_scan(T v, T *sh, T &total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nwarps = (blockDim.x + 31) >> 5;
+    const T incl = warp_incl_scan(v, lane);
+    __syncthreads();
+    if (lane == 31) sh[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const T w = lane < nwarps ? sh[lane] : T(0);
+        const T wi = warp_incl_scan(w, lane);
+        sh[lane] = wi - w;
+        if (lane == 31) sh[32] = wi;
+    }
+    __syncthreads();
+    total = sh[32];
+    return sh[warp] + incl - v;
+}
+
+template <typename T>
+__device__ __forceinline__ T block_sum(T v, T *sh) {
+    T total;
+    block_excl_scan(v, sh, total);
+    return total;
+}
+
+__global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p) {
+    constexpr int kMaxItems = kMaxCanvas / kScoreThreads;
+    __shared__ float shf[33];
+    __shared__ int shi[33];
+    __shared__ int first_reject;
+    __shared__ unsigned long long best_fb;
+
+    const int b = blockIdx.x;
+    const int N = p.N;
+    const int nmt = p.meta[kMetaMasked];
+    const int K = p.K;
+    const float tau = p.tau[b], beta = p.budget[b];
+    const int items = (N + blockDim.x - 1) / blockDim.x;
+    const int i0 = threadIdx.x * items;
+    uint8_t *mask = p.mask + static_cast<size_t>(b) * N;
+
+    bool masked[kMaxItems], cand[kMaxItems], high[kMaxItems];
+    int y[kMaxItems];
+    float conf[kMaxItems], H[kMaxItems];
+
+    int n_masked = 0, n_cand = 0;
+    float local_q = 0.f;
+#pragma unroll
+    for (int j = 0; j < kMaxItems; ++j) {
+        masked[j] = cand[j] = high[j] = false;
+        y[j] = -1;
+        conf[j] = H[j] = 0.f;
+        const int i = i0 + j;
+        if (j >= items || i >= N) continue;
+        const size_t pos = static_cast<size_t>(b) * N + i;
+        masked[j] = mask[i] != 0;
+        int ki = 0;
+        float r = 0.f, s = 0.f;
+        if (masked[j]) {
+            const int q = p.q_of_pos[pos];
+            const size_t last = static_cast<size_t>(K - 1) * nmt + q;
+            y[j] = p.row_arg[last];
+            conf[j] = p.row_pmax[last];
+            H[j] = p.row_H[last];
+            ki = 1;
+            float peak = conf[j];
+            for (int k = K - 2; k >= 0; --k) {
+                const size_t rk = static_cast<size_t>(k) * nmt + q;
+                if (p.row_arg[rk] != y[j]) break;
+                ++ki;
+                peak = fmaxf(peak, p.row_pmax[rk]);
+            }
+            r = peak - conf[j];
+            s = static_cast<float>(min(ki, p.k_max)) - p.w * r;
+            high[j] = conf[j] >= tau;
+            cand[j] = high[j] || (conf[j] >= p.theta_c && conf[j] < tau && s >= p.theta_s);
+            ++n_masked;
+            n_cand += cand[j];
+            if (!cand[j]) local_q += H[j];
+            if (p.dbg.layer_argmax || p.dbg.layer_pmax) {
+                for (int k = 0; k < K; ++k) {
+                    const size_t rk = static_cast<size_t>(k) * nmt + q;
+                    const size_t o = (static_cast<size_t>(k) * p.B) * N + pos;
+                    if (p.dbg.layer_argmax) p.dbg.layer_argmax[o] = p.row_arg[rk];
+                    if (p.dbg.layer_pmax) p.dbg.layer_pmax[o] = p.row_pmax[rk];
+                }
+            }
+        } else if (p.dbg.layer_argmax || p.dbg.layer_pmax) {
+            for (int k = 0; k < K; ++k) {
+                const size_t o = (static_cast<size_t>(k) * p.B) * N + pos;
+                if (p.dbg.layer_argmax) p.dbg.layer_argmax[o] = -1;
+                if (p.dbg.layer_pmax) p.dbg.layer_pmax[o] = 0.f;
+            }
+        }
+        if (p.dbg.conf) p.dbg.conf[pos] = masked[j] ? conf[j] : 0.f;
+        if (p.dbg.entropy) p.dbg.entropy[pos] = masked[j] ? H[j] : 0.f;
+        if (p.dbg.persist) p.dbg.persist[pos] = ki;
+        if (p.dbg.drop) p.dbg.drop[pos] = r;
+        if (p.dbg.stability) p.dbg.stability[pos] = masked[j] ? s : 0.f;
+        if (p.dbg.candidate) p.dbg.candidate[pos] = cand[j];
+    }
+
+    // ------------------------------------------- entropy of masked non-candidates, scanned
+    float q_total;
+    float q = block_excl_scan(local_q, shf, q_total);
+    if (threadIdx.x == 0) first_reject = N;
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < kMaxItems; ++j) {
+        if (j >= items || i0 + j >= N) break;
+        if (cand[j] && q > beta) {
+            atomicMin(&first_reject, i0 + j);
+            break;
+        }
+        if (masked[j] && !cand[j]) q += H[j];
+    }
+    __syncthreads();
+    const int reject_at = first_reject;
+
+    int n_acc = 0, n_high = 0;
+#pragma unroll
+    for (int j = 0; j < kMaxItems; ++j) {
+        const bool acc = cand[j] && (i0 + j) < reject_at;
+        n_acc += acc;
+        n_high += acc && high[j];
+    }
+    int dummy;
+    const int total_masked = block_sum(n_masked, shi);
+    const int total_acc = block_sum(n_acc, shi);
+    const int total_cand = block_sum(n_cand, shi);
+    const int total_high = block_sum(n_high, shi);
+
+    // ------------------------------------------------------------------------ fallback
+    int fb_pos = -1;
+    if (total_acc == 0 && total_masked > 0) {
+        int rank = block_excl_scan(n_masked, shi, dummy);
+        if (threadIdx.x == 0) best_fb = 0ull;
+        __syncthreads();
+        unsigned long long mine = 0ull;
+#pragma unroll
+        for (int j = 0; j < kMaxItems; ++j) {
+            if (!masked[j]) continue;
+            if (rank < p.window) {
+                // c >= 0: its bit pattern orders like the value; ties -> lowest position
+                const unsigned long long key =
+                    (static_cast<unsigned long long>(__float_as_uint(conf[j])) << 32) |
+                    static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<unsigned>(i0 + j));
+                mine = key > mine ? key : mine;
+            }
+            ++rank;
+        }
+        if (mine) atomicMax(&best_fb, mine);
+        __syncthreads();
+        fb_pos = static_cast<int>(0xFFFFFFFFu - static_cast<unsigned>(best_fb & 0xFFFFFFFFull));
+    }
+
+    // ------------------------------------------------------------------------- outputs
+#pragma unroll
+    for (int j = 0; j < kMaxItems; ++j) {
+        const int i = i0 + j;
+        if (j >= items || i >= N) break;
+        const size_t pos = static_cast<size_t>(b) * N + i;
+        const bool commit = (cand[j] && i < reject_at) || i == fb_pos;
+        p.out_commit[pos] = commit ? 1 : 0;
+        if (commit) {
+            p.out_token[pos] = y[j];
+            mask[i] = 0;
+        }
+    }
+    if (threadIdx.x == 0) {
+        rpd_stats st;
+        st.n_masked = total_masked;
+        st.n_candidates = total_cand;
+        st.n_high_conf = total_high;
+        st.n_stability = total_acc - total_high;
+        st.n_committed = total_acc + (fb_pos >= 0 ? 1 : 0);
+        st.fallback_used = fb_pos >= 0 ? 1 : 0;
+        st.fallback_pos = fb_pos;
+        st.status = p.meta[kMetaStatus];
+        p.out_stats[b] = st;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_merge(const MergeParams &p, int grid, cudaStream_t s) {
+    k_merge<<<grid, 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s) {
+    const int threads = p.N >= kScoreThreads ? kScoreThreads : ((p.N + 31) / 32) * 32;
+    k_score_commit<<<p.B, threads, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace rpd

@@ -1,0 +1,499 @@
+// rpd_host.cu - the C ABI of include/rpd.h: context, argument checks, scratch, TMA
+// descriptors and the launch sequence of one commit step.
+//
+// Step = k_compact -> k_gather_norm -> k_head_stats -> k_merge -> k_score_commit, all on
+// the context's stream, sized from device-resident counts (nothing is read back
+// mid-step).  Scratch is owned by the context and sized for the largest B*N seen.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "rpd_internal.h"
+
+using namespace rpd;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+    return fail(e == cudaErrorMemoryAllocation ? RPD_ERR_OUT_OF_MEMORY : RPD_ERR_CUDA, "%s: %s",
+                what, cudaGetErrorString(e));
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+// Row-major bf16 matrix [rows][cols] -> 2-D tensor map with a (64 x box_rows) box and
+// 128-byte swizzling; out-of-range elements read as zero.
+int encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,
+                   uint32_t box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(RPD_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(RPD_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return RPD_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+struct rpd_ctx {
+    int d = 0, V = 0, K = 0;
+    float eps = 0.f;
+    int device = 0, num_sms = 0;
+    const void *W = nullptr, *g = nullptr;
+    rpd_rule rule{0.6f, 3.5f, 15.0f, 6, 32};
+    cudaStream_t stream = nullptr;
+    rpd_debug dbg{};
+
+    // scratch, sized for cap_bn = B*N positions
+    int cap_bn = 0, cap_b = 0, cap_rows = 0, max_splits = 0;
+    __nv_bfloat16 *u = nullptr;
+    float *inv_rms = nullptr;
+    float4 *partials = nullptr;
+    int32_t *row_arg = nullptr;
+    float *row_pmax = nullptr, *row_H = nullptr;
+    int32_t *q_of_pos = nullptr, *pos_of_q = nullptr, *canvas_off = nullptr, *meta = nullptr;
+    CUtensorMap tmU{}, tmW{};
+
+    // host-buffer entry point staging
+    size_t stage_bytes = 0;
+    uint8_t *stage = nullptr;
+
+    // profiling
+    bool profile = false;
+    std::vector<cudaEvent_t> ev_pool;
+    std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_rec;
+    size_t ev_next = 0;
+
+    void free_scratch() {
+        void *ptrs[] = {u, inv_rms, partials, row_arg, row_pmax, row_H, q_of_pos, pos_of_q,
+                        canvas_off, meta};
+        for (void *p : ptrs)
+            if (p) cudaFree(p);
+        u = nullptr;
+        inv_rms = nullptr;
+        partials = nullptr;
+        row_arg = nullptr;
+        row_pmax = row_H = nullptr;
+        q_of_pos = pos_of_q = canvas_off = meta = nullptr;
+        cap_bn = cap_b = cap_rows = 0;
+    }
+};
+
+namespace {
+
+int ensure_scratch(rpd_ctx *c, int B, int N) {
+    const long long bn = static_cast<long long>(B) * N;
+    if (bn <= c->cap_bn && B <= c->cap_b) return RPD_OK;
+    const int new_bn = static_cast<int>(std::max<long long>(bn, c->cap_bn));
+    const int new_b = std::max(B, c->cap_b);
+    long long rows = static_cast<long long>(c->K) * new_bn;
+    rows = ((rows + kTileM - 1) / kTileM) * kTileM;
+    if (rows < kTileM) rows = kTileM;
+    if (rows > (1ll << 30)) return fail(RPD_ERR_UNSUPPORTED, "too many projected rows (%lld)", rows);
+    cudaError_t e = cudaStreamSynchronize(c->stream);  // no step may still use old scratch
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    c->free_scratch();
+    const int num_n = (c->V + kTileN - 1) / kTileN;
+    c->max_splits = std::min(num_n, 2 * c->num_sms);
+    struct {
+        void **p;
+        size_t bytes;
+    } allocs[] = {
+        {reinterpret_cast<void **>(&c->u), static_cast<size_t>(rows) * c->d * 2},
+        {reinterpret_cast<void **>(&c->inv_rms), static_cast<size_t>(rows) * 4},
+        {reinterpret_cast<void **>(&c->partials), static_cast<size_t>(rows) * c->max_splits * 16},
+        {reinterpret_cast<void **>(&c->row_arg), static_cast<size_t>(rows) * 4},
+        {reinterpret_cast<void **>(&c->row_pmax), static_cast<size_t>(rows) * 4},
+        {reinterpret_cast<void **>(&c->row_H), static_cast<size_t>(rows) * 4},
+        {reinterpret_cast<void **>(&c->q_of_pos), static_cast<size_t>(new_bn) * 4},
+        {reinterpret_cast<void **>(&c->pos_of_q), static_cast<size_t>(new_bn) * 4},
+        {reinterpret_cast<void **>(&c->canvas_off), static_cast<size_t>(new_b + 1) * 4},
+        {reinterpret_cast<void **>(&c->meta), kMetaWords * 4},
+    };
+    for (auto &a : allocs) {
+        e = cudaMalloc(a.p, a.bytes);
+        if (e != cudaSuccess) {
+            c->free_scratch();
+            return cuda_fail(e, "cudaMalloc(scratch)");
+        }
+    }
+    // the head operand rows past the live count are read by the last tile: keep them finite
+    e = cudaMemsetAsync(c->u, 0, static_cast<size_t>(rows) * c->d * 2, c->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->meta, 0, kMetaWords * 4, c->stream);
+    if (e != cudaSuccess) {
+        c->free_scratch();
+        return cuda_fail(e, "cudaMemsetAsync(scratch)");
+    }
+    c->cap_bn = new_bn;
+    c->cap_b = new_b;
+    c->cap_rows = static_cast<int>(rows);
+    return encode_bf16_2d(&c->tmU, c->u, static_cast<uint64_t>(rows), c->d, kTileM);
+}
+
+cudaEvent_t take_event(rpd_ctx *c) {
+    if (c->ev_next == c->ev_pool.size()) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        c->ev_pool.push_back(e);
+    }
+    return c->ev_pool[c->ev_next++];
+}
+
+struct KernelTimer {
+    rpd_ctx *c;
+    int kernel;
+    cudaEvent_t a = nullptr, b = nullptr;
+    KernelTimer(rpd_ctx *ctx, int k) : c(ctx), kernel(k) {
+        if (c->profile) {
+            a = take_event(c);
+            b = take_event(c);
+            if (a && b) cudaEventRecord(a, c->stream);
+        }
+    }
+    ~KernelTimer() {
+        if (a && b) {
+            cudaEventRecord(b, c->stream);
+            c->ev_rec.push_back({kernel, {a, b}});
+        }
+    }
+};
+
+int check_rule(const rpd_rule &r) {
+    if (!(r.theta_c >= 0.f) || !std::isfinite(r.theta_c))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "theta_c must be finite and >= 0");
+    if (std::isnan(r.theta_s)) return fail(RPD_ERR_INVALID_ARGUMENT, "theta_s is NaN");
+    if (!(r.w >= 0.f) || !std::isfinite(r.w))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "w must be finite and >= 0");
+    if (r.k_max < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "k_max must be >= 1");
+    if (r.window < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "window must be >= 1");
+    return RPD_OK;
+}
+
+int check_call(const rpd_ctx *c, float tau, float budget) {
+    if (!(tau > 0.f && tau <= 1.f)) return fail(RPD_ERR_INVALID_ARGUMENT, "tau must be in (0, 1]");
+    if (!(c->rule.theta_c < tau))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "theta_c (%g) must be below tau (%g)",
+                    (double)c->rule.theta_c, (double)tau);
+    if (!(budget >= 0.f)) return fail(RPD_ERR_INVALID_ARGUMENT, "budget must be >= 0 (got %g)",
+                                      (double)budget);
+    return RPD_OK;
+}
+
+int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const float *tau,
+             const float *budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (!c->W || !c->g) return fail(RPD_ERR_NO_HEAD, "rpd_set_head has not been called");
+    if (B < 1 || B > kMaxBatch) return fail(RPD_ERR_INVALID_ARGUMENT, "B must be in [1, %d]", kMaxBatch);
+    if (N < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be >= 0");
+    if (N > kMaxCanvas) return fail(RPD_ERR_UNSUPPORTED, "N must be <= %d", kMaxCanvas);
+    if (!tau || !budget) return fail(RPD_ERR_INVALID_ARGUMENT, "null tau/budget");
+    for (int b = 0; b < B; ++b) {
+        int rc = check_call(c, tau[b], budget[b]);
+        if (rc) return rc;
+    }
+    if (N == 0) return RPD_OK;
+    if (!hidden || !mask || !out_commit || !out_token || !out_stats)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
+    if (!aligned16(hidden)) return fail(RPD_ERR_INVALID_ARGUMENT, "hidden must be 16-byte aligned");
+    int rc = ensure_scratch(c, B, N);
+    if (rc) return rc;
+
+    const int bn = B * N;
+    const int num_n = (c->V + kTileN - 1) / kTileN;
+    const int grid_head = c->num_sms;
+    cudaError_t e;
+    {
+        KernelTimer t(c, 0);
+        CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
+                         num_n, grid_head, c->max_splits};
+        e = launch_compact(cp, c->stream);
+        if (e == cudaSuccess) {
+            NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
+                          static_cast<const __nv_bfloat16 *>(c->g), c->pos_of_q, c->meta, c->u,
+                          c->inv_rms, bn, c->d, c->eps};
+            e = launch_gather_norm(np, c->num_sms * 8, c->stream);
+        }
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "gather/norm launch");
+    {
+        KernelTimer t(c, 1);
+        HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits};
+        e = launch_head_stats(c->tmU, c->tmW, hp, grid_head, c->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "head statistics launch");
+    {
+        KernelTimer t(c, 2);
+        MergeParams mp{c->partials, c->meta, c->row_arg, c->row_pmax, c->row_H, c->max_splits};
+        e = launch_merge(mp, c->num_sms * 8, c->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+    {
+        KernelTimer t(c, 3);
+        ScoreParams sp{};
+        sp.mask = mask;
+        sp.q_of_pos = c->q_of_pos;
+        sp.canvas_off = c->canvas_off;
+        sp.meta = c->meta;
+        sp.row_arg = c->row_arg;
+        sp.row_pmax = c->row_pmax;
+        sp.row_H = c->row_H;
+        sp.out_commit = out_commit;
+        sp.out_token = out_token;
+        sp.out_stats = out_stats;
+        sp.dbg = c->dbg;
+        sp.B = B;
+        sp.N = N;
+        sp.K = c->K;
+        sp.theta_c = c->rule.theta_c;
+        sp.theta_s = c->rule.theta_s;
+        sp.w = c->rule.w;
+        sp.k_max = c->rule.k_max;
+        sp.window = c->rule.window;
+        for (int b = 0; b < B; ++b) {
+            sp.tau[b] = tau[b];
+            sp.budget[b] = budget[b];
+        }
+        e = launch_score_commit(sp, c->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "score/commit launch");
+    return RPD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *rpd_last_error(void) { return g_last_error.c_str(); }
+
+const char *rpd_version(void) { return "rpd-gb300 0.1 (sm_103a, tcgen05 head statistics)"; }
+
+rpd_ctx *rpd_create(int d, int V, int K, float eps) {
+    if (d < 64 || d % 8 != 0) {
+        fail(RPD_ERR_INVALID_ARGUMENT, "d must be a multiple of 8 and >= 64 (got %d)", d);
+        return nullptr;
+    }
+    if (V < kTileN) {
+        fail(RPD_ERR_UNSUPPORTED, "V must be >= %d (got %d)", kTileN, V);
+        return nullptr;
+    }
+    if (K < 1 || K > 64) {
+        fail(RPD_ERR_INVALID_ARGUMENT, "K must be in [1, 64] (got %d)", K);
+        return nullptr;
+    }
+    if (!(eps >= 0.f) || !std::isfinite(eps)) {
+        fail(RPD_ERR_INVALID_ARGUMENT, "eps must be finite and >= 0");
+        return nullptr;
+    }
+    rpd_ctx *c = new rpd_ctx();
+    c->d = d;
+    c->V = V;
+    c->K = K;
+    c->eps = eps;
+    cudaError_t e = cudaGetDevice(&c->device);
+    if (e == cudaSuccess)
+        e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess) {
+        cuda_fail(e, "device query");
+        delete c;
+        return nullptr;
+    }
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, c->device);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, c->device);
+    if (major != 10 || minor != 3) {
+        fail(RPD_ERR_UNSUPPORTED, "device is sm_%d%d; this library is built for sm_103a", major, minor);
+        delete c;
+        return nullptr;
+    }
+    return c;
+}
+
+int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
+    if (!c || !W_head || !g_norm) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    if (!aligned16(W_head) || !aligned16(g_norm))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "W_head and g_norm must be 16-byte aligned");
+    CUtensorMap m;
+    int rc = encode_bf16_2d(&m, W_head, static_cast<uint64_t>(c->V), c->d, kTileN);
+    if (rc) return rc;
+    c->tmW = m;
+    c->W = W_head;
+    c->g = g_norm;
+    return RPD_OK;
+}
+
+int rpd_set_rule(rpd_ctx *c, const rpd_rule *r) {
+    if (!c || !r) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    int rc = check_rule(*r);
+    if (rc) return rc;
+    c->rule = *r;
+    return RPD_OK;
+}
+
+int rpd_get_rule(const rpd_ctx *c, rpd_rule *r) {
+    if (!c || !r) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    *r = c->rule;
+    return RPD_OK;
+}
+
+int rpd_set_stream(rpd_ctx *c, void *stream) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    c->stream = static_cast<cudaStream_t>(stream);
+    return RPD_OK;
+}
+
+int rpd_reserve(rpd_ctx *c, int B, int N) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (B < 1 || B > kMaxBatch || N < 1 || N > kMaxCanvas)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "reserve: B in [1,%d], N in [1,%d]", kMaxBatch, kMaxCanvas);
+    return ensure_scratch(c, B, N);
+}
+
+int rpd_set_debug(rpd_ctx *c, const rpd_debug *dbg) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (dbg)
+        c->dbg = *dbg;
+    else
+        c->dbg = rpd_debug{};
+    return RPD_OK;
+}
+
+int rpd_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float tau, float budget,
+             uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
+    return run_step(c, hidden, mask, 1, N, &tau, &budget, out_commit, out_token, out_stats);
+}
+
+int rpd_step_batched(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const float *tau,
+                     const float *budget, uint8_t *out_commit, int32_t *out_token,
+                     rpd_stats *out_stats) {
+    return run_step(c, hidden, mask, B, N, tau, budget, out_commit, out_token, out_stats);
+}
+
+int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float tau, float budget,
+                  uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (N < 0 || N > kMaxCanvas) return fail(RPD_ERR_INVALID_ARGUMENT, "N out of range");
+    if (N == 0) return run_step(c, nullptr, nullptr, 1, 0, &tau, &budget, nullptr, nullptr, nullptr);
+    if (!hidden || !mask || !out_commit || !out_token || !out_stats)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
+    const size_t hid = static_cast<size_t>(c->K) * N * c->d * 2;
+    const size_t off_mask = (hid + 255) & ~size_t(255);
+    const size_t off_commit = off_mask + ((N + 255) & ~255);
+    const size_t off_token = off_commit + ((N + 255) & ~255);
+    const size_t off_stats = off_token + ((static_cast<size_t>(N) * 4 + 255) & ~size_t(255));
+    const size_t need = off_stats + 256;
+    if (need > c->stage_bytes) {
+        cudaError_t e = cudaStreamSynchronize(c->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+        if (c->stage) cudaFree(c->stage);
+        c->stage = nullptr;
+        c->stage_bytes = 0;
+        e = cudaMalloc(&c->stage, need);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(staging)");
+        c->stage_bytes = need;
+    }
+    uint8_t *d_hidden = c->stage;
+    uint8_t *d_mask = c->stage + off_mask;
+    uint8_t *d_commit = c->stage + off_commit;
+    int32_t *d_token = reinterpret_cast<int32_t *>(c->stage + off_token);
+    rpd_stats *d_stats = reinterpret_cast<rpd_stats *>(c->stage + off_stats);
+    cudaError_t e = cudaMemcpyAsync(d_hidden, hidden, hid, cudaMemcpyHostToDevice, c->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(d_mask, mask, N, cudaMemcpyHostToDevice, c->stream);
+    // tokens are written only where committed: start from the caller's canvas
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(d_token, out_token, static_cast<size_t>(N) * 4, cudaMemcpyHostToDevice,
+                            c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "host->device copy");
+    int rc = run_step(c, d_hidden, d_mask, 1, N, &tau, &budget, d_commit, d_token, d_stats);
+    if (rc) return rc;
+    e = cudaMemcpyAsync(mask, d_mask, N, cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(out_commit, d_commit, N, cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(out_token, d_token, static_cast<size_t>(N) * 4, cudaMemcpyDeviceToHost,
+                            c->stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(out_stats, d_stats, sizeof(rpd_stats), cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "device->host copy");
+    return RPD_OK;
+}
+
+int rpd_profile_enable(rpd_ctx *c, int enable) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    c->profile = enable != 0;
+    return RPD_OK;
+}
+
+int rpd_kernel_times(rpd_ctx *c, double *ms, int64_t *launches, int reset) {
+    if (!c || !ms || !launches) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    for (int k = 0; k < RPD_NUM_KERNELS; ++k) {
+        ms[k] = 0.0;
+        launches[k] = 0;
+    }
+    for (auto &r : c->ev_rec) {
+        cudaError_t e = cudaEventSynchronize(r.second.second);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+        float t = 0.f;
+        e = cudaEventElapsedTime(&t, r.second.first, r.second.second);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+        ms[r.first] += t;
+        launches[r.first] += 1;
+    }
+    if (reset) {
+        c->ev_rec.clear();
+        c->ev_next = 0;
+    }
+    return RPD_OK;
+}
+
+void rpd_destroy(rpd_ctx *c) {
+    if (!c) return;
+    cudaStreamSynchronize(c->stream);
+    c->free_scratch();
+    if (c->stage) cudaFree(c->stage);
+    for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
+    delete c;
+}
+
+}  // extern "C"

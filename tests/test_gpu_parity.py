@@ -1,0 +1,262 @@
+"""Parity of the CUDA commit step with the CPU oracle, through the C ABI, on cuda:0.
+
+Tolerances and the near-threshold exemption are stated in ``tests/parity.py``.
+Small cases compare every output element by element; the full-size LLaDA-8B and
+Dream-7B head shapes run the oracle over every projected row (fp64 BLAS).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import workloads as WL
+from oracle import rpd_oracle as O
+from tests.gpu_util import GpuRunner, bits
+from tests.parity import compare_step
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # collected on CPU machines, never run there
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+
+def oracle_step(case, hidden=None, mask=None, tau=None, budget=None, rule=None):
+    hidden = case["hidden"] if hidden is None else hidden
+    mask = case["mask"] if mask is None else mask
+    return O.rpd_step(bits(hidden), mask.numpy(), bits(case["g"]), bits(case["W"]), case["eps"],
+                      case["tau"] if tau is None else tau,
+                      case["budget"] if budget is None else budget,
+                      case["rule"] if rule is None else rule)
+
+
+def small_case(seed, K=3, N=64, d=256, V=4096, w_std=0.08, sigma=None, flip=0.1, a=None,
+               mask_frac=1.0, tau=0.9, budget=1.0, rule="llada", b=None):
+    """Calibrated small workload: U-shaped signal whose canvas ends are confident."""
+    W, g = WL.make_head(V, d, seed, w_std=w_std)
+    b = WL.u_profile(N, 0.5, 3.0) if b is None else b
+    if sigma is None:
+        sigma = WL.calibrated_sigma(V, d, w_std, b_max=float(b.max()))
+    cv = WL.make_hidden(W, K, N, seed + 1000, b, sigma, flip_frac=flip, a=a)
+    mask = torch.ones(N, dtype=torch.uint8) if mask_frac >= 1.0 else \
+        WL.uniform_fraction_mask(N, mask_frac, seed + 5)
+    return dict(W=W, g=g, hidden=cv.hidden, mask=mask, K=K, N=N, d=d, V=V, eps=1e-6, tau=tau,
+                budget=budget, rule=rule)
+
+
+def run_and_compare(case, rule=None, tau=None, budget=None, mask=None):
+    runner = GpuRunner(case["W"], case["g"], case["K"], case["eps"],
+                       rule=case["rule"] if rule is None else rule)
+    try:
+        m = case["mask"] if mask is None else mask
+        got = runner.step(case["hidden"], m, case["tau"] if tau is None else tau,
+                          case["budget"] if budget is None else budget)
+        ref = oracle_step(case, mask=m, tau=tau, budget=budget, rule=rule)
+        rep = compare_step(ref, got)
+        return ref, got, rep
+    finally:
+        runner.close()
+
+
+# ------------------------------------------------------------------------- small cases
+
+def test_tiny_literal_takes_fallback():
+    """The literal tiny workload (N=64, K=3, d=256, V=4096): no confident position exists,
+    so every step is the fallback commit of the most confident early position."""
+    case = WL.tiny_step(seed=1, calibrated=False)
+    ref, got, rep = run_and_compare(case)
+    assert got["stats"]["fallback_used"] == 1 and got["stats"]["n_committed"] == 1
+    assert np.nanmax(ref.conf) < 0.05
+    print(rep)
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3, 4])
+def test_tiny_calibrated(seed):
+    case = WL.tiny_step(seed=seed, calibrated=True)
+    ref, got, rep = run_and_compare(case)
+    print(rep)
+
+
+def test_paths_are_exercised():
+    """Across a few calibrated seeds the budget holds candidates back, high-confidence and
+    stability admissions both commit, and flipped positions have persistence 1."""
+    held = high = stab = 0
+    for seed in range(10, 16):
+        case = small_case(seed, K=4, N=96, a=torch.ones(4), flip=0.15)
+        ref, got, rep = run_and_compare(case, rule=dict(O.RULES["llada"], theta_s=2.0))
+        held += int(ref.cand.sum() - len(ref.accepted))
+        high += got["stats"]["n_high_conf"]
+        stab += got["stats"]["n_stability"]
+    assert held > 0 and high > 0 and stab > 0, (held, high, stab)
+
+
+@pytest.mark.parametrize("d,V,K,N,frac", [
+    (200, 1000, 2, 77, 0.7),     # ragged K-block (200 = 3*64+8) and vocabulary tile (1000)
+    (128, 4100, 5, 300, 1.0),    # 1500 rows: 12 row tiles, last one ragged; V ragged
+    (64, 256, 1, 33, 1.0),       # single vocabulary tile, K = 1
+    (4096, 1280, 3, 50, 0.5),    # LLaDA hidden size, 64 K-blocks
+])
+def test_ragged_shapes(d, V, K, N, frac):
+    case = small_case(7 + d + V, K=K, N=N, d=d, V=V, w_std=0.08, mask_frac=frac)
+    ref, got, rep = run_and_compare(case)
+    print(rep)
+
+
+def test_stability_route_with_drops():
+    """Flat layer ramp with explicit theta_s: persistence is long and drops small but
+    nonzero, so the stability route admits and rejects on the drop penalty."""
+    case = small_case(31, K=6, N=128, a=torch.tensor([1.0, 0.95, 1.05, 1.0, 0.97, 1.0]), flip=0.1)
+    rule = dict(theta_c=0.6, theta_s=4.5, w=15.0, k_max=6, window=32)
+    ref, got, rep = run_and_compare(case, rule=rule, budget=50.0)
+    m = ref.masked
+    assert np.any(ref.drop[m] > 0.001)
+    print(rep, "stability commits", got["stats"]["n_stability"])
+
+
+@pytest.mark.parametrize("tau,budget", [(0.9, 0.0), (0.9, math.inf), (1.0, 1.0), (0.61, 4.0)])
+def test_threshold_extremes(tau, budget):
+    case = small_case(41, K=3, N=80)
+    run_and_compare(case, tau=tau, budget=budget)
+
+
+def test_fallback_window_counts_masked_positions():
+    case = small_case(43, K=3, N=100, mask_frac=0.4, w_std=0.02, sigma=1.0)
+    rule = dict(O.RULES["llada"], window=3)
+    ref, got, rep = run_and_compare(case, rule=rule)
+    assert got["stats"]["fallback_used"] == 1
+    first3 = np.nonzero(ref.masked)[0][:3]
+    assert got["stats"]["fallback_pos"] in first3
+
+
+def test_empty_and_single_masks():
+    case = small_case(45, K=3, N=40)
+    runner = GpuRunner(case["W"], case["g"], 3)
+    try:
+        none = torch.zeros(40, dtype=torch.uint8)
+        got = runner.step(case["hidden"], none, 0.9, 1.0)
+        assert got["commit"].sum() == 0 and np.all(got["new_mask"] == 0)
+        assert got["stats"]["n_masked"] == 0 and got["stats"]["n_committed"] == 0
+        assert got["stats"]["fallback_pos"] == -1 and got["stats"]["status"] == 0
+        assert np.all(got["token"] == -5)  # tokens untouched where nothing commits
+        one = torch.zeros(40, dtype=torch.uint8)
+        one[17] = 1
+        got = runner.step(case["hidden"], one, 0.9, 1.0)
+        ref = oracle_step(case, mask=one)
+        compare_step(ref, got)
+        assert got["commit"][17] == 1 and got["stats"]["n_committed"] == 1
+        # N = 1
+        h1 = case["hidden"][:, :1].contiguous()
+        got = runner.step(h1, torch.ones(1, dtype=torch.uint8), 0.9, 1.0)
+        assert got["commit"][0] == 1
+    finally:
+        runner.close()
+
+
+def test_batched_matches_per_canvas_oracle():
+    K, N, d, V, B = 3, 120, 256, 2048, 4
+    W, g = WL.make_head(V, d, 51, w_std=0.08)
+    hidden = torch.empty(K, B, N, d, dtype=torch.bfloat16)
+    masks = torch.empty(B, N, dtype=torch.uint8)
+    for b in range(B):
+        cv = WL.make_hidden(W, K, N, 600 + b, WL.u_profile(N, 0.5, 3.0),
+                              WL.calibrated_sigma(V, d, 0.08, 3.0), flip_frac=0.1)
+        hidden[:, b] = cv.hidden
+        masks[b] = WL.uniform_fraction_mask(N, [1.0, 0.5, 0.0, 0.9][b], 700 + b)
+    taus, budgets = [0.9, 0.8, 0.9, 0.95], [1.0, 3.0, 1.0, 0.5]
+    runner = GpuRunner(W, g, K)
+    try:
+        outs = runner.step_batched(hidden, masks, taus, budgets)
+    finally:
+        runner.close()
+    for b in range(B):
+        ref = O.rpd_step(bits(hidden[:, b]), masks[b].numpy(), bits(g), bits(W), 1e-6, taus[b],
+                         budgets[b], "llada")
+        compare_step(ref, outs[b])
+    assert outs[2]["stats"]["n_masked"] == 0
+
+
+def test_host_entry_point_matches_device():
+    case = small_case(61, K=3, N=64)
+    runner = GpuRunner(case["W"], case["g"], 3)
+    try:
+        dev = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
+        hid = case["hidden"].contiguous().pin_memory()
+        mask = case["mask"].clone().pin_memory()
+        commit = torch.zeros(64, dtype=torch.uint8).pin_memory()
+        token = torch.full((64,), -5, dtype=torch.int32).pin_memory()
+        stats = torch.zeros(8, dtype=torch.int32).pin_memory()
+        runner.ctx.set_debug()
+        runner.ctx.step_host(hid, mask, 0.9, 1.0, commit, token, stats)
+        assert np.array_equal(commit.numpy(), dev["commit"])
+        assert np.array_equal(mask.numpy(), dev["new_mask"])
+        sel = dev["commit"] == 1
+        assert np.array_equal(token.numpy()[sel], dev["token"][sel])
+        assert np.all(token.numpy()[~sel] == -5)
+        assert runner.rpd.stats_dict(stats) == dev["stats"]
+    finally:
+        runner.close()
+
+
+def test_repeat_is_bit_identical():
+    case = small_case(71, K=4, N=200, d=512, V=3000)
+    runner = GpuRunner(case["W"], case["g"], 4)
+    try:
+        a = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
+        b = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
+    finally:
+        runner.close()
+    for k in a:
+        if k == "stats":
+            assert a[k] == b[k]
+        else:
+            assert np.array_equal(a[k], b[k]), k
+
+
+def test_invalid_arguments_on_gpu():
+    import paper_2609_36452_gb300 as rpd
+    ctx = rpd.Rpd(256, 4096, 3)
+    dev = torch.device("cuda:0")
+    h = torch.zeros(3, 8, 256, dtype=torch.bfloat16, device=dev)
+    m = torch.ones(8, dtype=torch.uint8, device=dev)
+    c = torch.zeros(8, dtype=torch.uint8, device=dev)
+    t = torch.zeros(8, dtype=torch.int32, device=dev)
+    s = torch.zeros(8, dtype=torch.int32, device=dev)
+    with pytest.raises(rpd.RpdError) as e:
+        ctx.step(h, m, 0.9, 1.0, c, t, s)
+    assert e.value.code == rpd.RPD_ERR_NO_HEAD
+    W = torch.zeros(4096, 256, dtype=torch.bfloat16, device=dev)
+    g = torch.ones(256, dtype=torch.bfloat16, device=dev)
+    ctx.set_head(W, g)
+    for tau, budget in [(0.5, 1.0), (0.0, 1.0), (1.5, 1.0), (0.9, -1.0), (0.9, float("nan"))]:
+        with pytest.raises(rpd.RpdError) as e:
+            ctx.step(h, m, tau, budget, c, t, s)
+        assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+    with pytest.raises(rpd.RpdError) as e:
+        ctx.set_rule(0.6, 3.5, 15.0, 0, 32)
+    assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+    ctx.close()
+
+
+# ------------------------------------------------------------------ full-size head shapes
+
+@pytest.fixture(scope="module")
+def llada_head():
+    return WL.make_head(WL.LLADA_V, WL.LLADA_D, seed=2)
+
+
+def test_llada_first_step_full(llada_head):
+    """Batch 1, N=256 all masked, K=4, d=4096, V=126464 (1024 projected rows): every row
+    checked against the oracle."""
+    W, g = llada_head
+    case = WL.llada_first_step(seed=2, W=W, g=g)
+    ref, got, rep = run_and_compare(case)
+    print(rep, got["stats"])
+    assert got["stats"]["n_committed"] >= 1
+
+
+def test_dream_mid_decode_full():
+    """Batch 1, N=512, front-loaded 50% mask, K=4, d=3584, V=152064, tau 0.85, budget 2,
+    Dream rule profile."""
+    case = WL.dream_mid_decode(seed=3)
+    ref, got, rep = run_and_compare(case)
+    print(rep, got["stats"])

@@ -141,6 +141,16 @@ def uniform_fraction_mask(N: int, frac: float, seed: int) -> torch.Tensor:
     return m
 
 
+def calibrated_sigma(V: int, d: int, w_std: float, b_max: float, margin: float = 5.0) -> float:
+    """Signal scale putting the final-layer target logit at ``b_max`` a ``margin`` (nats)
+    above the log-partition of the noise logits.  With h = sigma*b*w_hat + n and
+    W ~ N(0, w_std), the target logit is about sigma*b*w_std*sqrt(d) and the V noise
+    logits are about N(0, (w_std*sqrt(d))^2), whose log-partition is
+    ln V + (w_std*sqrt(d))^2 / 2."""
+    s = w_std * math.sqrt(d)
+    return (math.log(V) + 0.5 * s * s + margin) / (b_max * s)
+
+
 # --------------------------------------------------------------------------------------
 # Named workloads.  Each returns a dict with the head, the hidden states, the mask(s) and
 # the per-call parameters; "rule" names the Table 4 profile (llada or dream).
@@ -151,14 +161,15 @@ def tiny_step(seed: int = 1, calibrated: bool = False):
 
     ``calibrated=False`` is the literal recipe (W ~ N(0, 0.02), sigma = 1), whose
     confidences stay near 1/V so every step takes the fallback commit.
-    ``calibrated=True`` widens the head to W ~ N(0, 0.08) and uses sigma = kappa*sqrt(d)
-    with kappa = 0.08 so that candidates, budget waits and fallbacks all occur.
+    ``calibrated=True`` widens the head to W ~ N(0, 0.08) and sets the signal so that the
+    final-layer target logit at the canvas ends sits 5 nats above the noise partition
+    (``calibrated_sigma``), so that candidates, budget waits and fallbacks all occur.
     """
     K, N, d, V = 3, 64, 256, 4096
     w_std = 0.08 if calibrated else 0.02
     W, g = make_head(V, d, seed, w_std=w_std)
     b = u_profile(N, 0.5, 3.0)
-    sigma = 0.08 * math.sqrt(d) if calibrated else 1.0
+    sigma = calibrated_sigma(V, d, w_std, b_max=3.0) if calibrated else 1.0
     cv = make_hidden(W, K, N, seed + 1000, b, sigma, flip_frac=0.1 if calibrated else 0.0)
     mask = torch.ones(N, dtype=torch.uint8)
     return dict(name="tiny", W=W, g=g, hidden=cv.hidden, mask=mask, K=K, N=N, d=d, V=V,
