@@ -108,10 +108,17 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def make_workload(rank: int):
+def make_workload(rank: int, masked: int = 0):
+    """The LLaDA first-step canvas; ``masked`` > 0 keeps only the last ``masked`` positions
+    masked (the few-rows, head-streaming regime at the end of a decode trajectory)."""
     import workloads as WL
     W, g = WL.make_head(WL.LLADA_V, WL.LLADA_D, seed=2)
     case = WL.llada_first_step(seed=2 + 97 * rank, W=W, g=g)
+    if masked:
+        m = torch.zeros(case["N"], dtype=torch.uint8)
+        m[case["N"] - masked:] = 1
+        case["mask"] = m
+        case["name"] = f"llada_tail_{masked}_masked"
     return case
 
 
@@ -190,7 +197,7 @@ def run_reference(args):
 
 
 def config_dict(case, R):
-    return {"workload": "llada_first_step", "batch": 1, "N": case["N"], "K": case["K"],
+    return {"workload": case["name"], "batch": 1, "N": case["N"], "K": case["K"],
             "d": case["d"], "V": case["V"], "rows": R, "tau": case["tau"], "budget": case["budget"],
             "rule": "llada (Table 4)", "signal_kappa": case.get("kappa"),
             "l2": "inputs larger than L2: the 1.04 GB head is streamed every step"}
@@ -205,7 +212,7 @@ def run_rpd(args):
         dist.init_process_group("nccl", device_id=dev)
     import paper_2609_36452_gb300 as rpd
 
-    case = make_workload(rank)
+    case = make_workload(rank, args.masked)
     K, N, d, V = case["K"], case["N"], case["d"], case["V"]
     R, flops, bytes_ = work_per_step(case)
     W = case["W"].to(dev)
@@ -266,6 +273,26 @@ def run_rpd(args):
     steps_s = world * args.steps / (ms_total / 1e3)
 
     # ---------------------------------------------------------------- end to end (host buffers)
+    e2e = None
+    if not args.no_e2e:
+        e2e = measure_e2e(ctx, case, args, world, barrier, dev)
+
+    if rank != 0:
+        ctx.close()
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st, world)
+    ctx.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def measure_e2e(ctx, case, args, world, barrier, dev):
+    """Same step through rpd_step_host: pinned host inputs copied in, results read back."""
+    N = case["N"]
     hid_h = case["hidden"].contiguous().pin_memory()
     mask_h0 = case["mask"].clone()
     mask_h = mask_h0.clone().pin_memory()
@@ -289,14 +316,12 @@ def run_rpd(args):
         e2e_s = float(t.item())
     h2d = hid_h.numel() * 2 + N + N * 4
     d2h = N + N + N * 4 + 32
+    return {"value": e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "api": "rpd_step_host (pinned host buffers)"}
 
-    if rank != 0:
-        ctx.close()
-        if world > 1:
-            import torch.distributed as dist
-            dist.destroy_process_group()
-        return
 
+def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st, world):
+    K = case["K"]
     peaks = load_peaks()
     head_ms, head_n = ktimes["head_stats"]
     head_avg_ms = head_ms / max(head_n, 1)
@@ -334,17 +359,12 @@ def run_rpd(args):
         "step_roofline_frac": step_roof,
         "kernels_ms": {k: (v[0] / max(v[1], 1)) for k, v in ktimes.items()},
         "cpu_baseline": cpu,
-        "e2e": {"value": e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "api": "rpd_step_host (pinned host buffers)"},
+        "e2e": e2e,
         "gpu_launches": 5 * args.steps,
         "clocks": clocks,
         "last_step_stats": st,
     }
     print(json.dumps(out))
-    ctx.close()
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
 
 
 def main():
@@ -357,6 +377,9 @@ def main():
     ap.add_argument("--ref-positions", type=int, default=8)
     ap.add_argument("--ref-seconds", type=float, default=150.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--masked", type=int, default=0,
+                    help="keep only the last N canvas positions masked (head-streaming regime)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
