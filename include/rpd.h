@@ -146,6 +146,29 @@ int rpd_profile_enable(rpd_ctx *ctx, int enable);
 int rpd_kernel_times(rpd_ctx *ctx, double *ms /*[RPD_NUM_KERNELS]*/,
                      int64_t *launches /*[RPD_NUM_KERNELS]*/, int reset);
 
+/* rpd_step for callers that cannot allocate device memory.  (The paper has no counterpart:
+ * this is a deployment variant of rpd_step.)  Some callers own every byte of device memory
+ * themselves - a serving engine that plans one fixed arena, a plugin running inside another
+ * framework's memory manager, code that must not allocate while its stream is captured - so
+ * a library that calls cudaMalloc on their behalf is not an option.  This entry point takes
+ * no context and allocates nothing: it runs the same kernels as rpd_step with its scratch in
+ * a static device array of this library (about 13 MiB, held on every GPU that loads the
+ * library until the process exits).  The caller passes every input and output.
+ *   W_head [V][d], g_norm [d], hidden [K][N][d]: bf16 device, 16-byte aligned;
+ *   rule: NULL for the LLaDA profile of Table 4; mask/out_commit/out_token/out_stats and
+ *   tau/budget as in rpd_step; stream: a cudaStream_t (NULL = legacy default stream).
+ * Limits: K*N <= 1024, N <= 1024, d <= 4096 (plus rpd_create's shape rules); larger sizes
+ * return RPD_ERR_UNSUPPORTED with a message naming the limit, before any work is enqueued.
+ * All calls on a device share the one scratch array, which keeps the previous call's
+ * contents (the step's count/status words are cleared at the start of every call): calls
+ * whose GPU work overlaps - concurrent host threads or different streams - race on it, so
+ * order them on one stream.  The first call on each device finds the array's device address
+ * (cudaGetSymbolAddress) and caches it; make that first call before any stream capture. */
+int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, int V, int K, float eps,
+                     const rpd_rule *rule, const void *hidden, uint8_t *mask, int N, float tau,
+                     float budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats,
+                     void *stream);
+
 /* Free the context and its scratch (not the borrowed head).  NULL is ignored. */
 void rpd_destroy(rpd_ctx *ctx);
 

@@ -16,7 +16,7 @@ __all__ = [
     "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
     "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_step",
-    "rpd_step_batched", "rpd_step_host", "rpd_profile_enable", "rpd_kernel_times",
+    "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_profile_enable", "rpd_kernel_times",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
 
@@ -83,6 +83,8 @@ def _load():
         "rpd_step": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_step_batched": (i32, [vp, vp, vp, i32, i32, vp, vp, vp, vp, vp]),
         "rpd_step_host": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
+        "rpd_step_noalloc": (i32, [vp, vp, i32, i32, i32, f32, ctypes.POINTER(RpdRule), vp, vp,
+                                   i32, f32, f32, vp, vp, vp, vp]),
         "rpd_profile_enable": (i32, [vp, i32]),
         "rpd_kernel_times": (i32, [vp, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_int64), i32]),
@@ -109,6 +111,7 @@ rpd_set_debug = lib.rpd_set_debug
 rpd_step = lib.rpd_step
 rpd_step_batched = lib.rpd_step_batched
 rpd_step_host = lib.rpd_step_host
+rpd_step_noalloc = lib.rpd_step_noalloc
 rpd_profile_enable = lib.rpd_profile_enable
 rpd_kernel_times = lib.rpd_kernel_times
 rpd_destroy = lib.rpd_destroy

@@ -13,7 +13,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "librpd.so")
-SOURCES = ["rpd_host.cu", "k_gather_norm.cu", "k_head_stats.cu", "k_merge_commit.cu"]
+SOURCES = ["rpd_host.cu", "k_gather_norm.cu", "k_head_stats.cu", "k_merge_commit.cu",
+           "rpd_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -303,6 +303,8 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
 
 }  // namespace
 
+void rpd::set_last_error(const char *msg) { g_last_error = msg ? msg : ""; }
+
 extern "C" {
 
 const char *rpd_last_error(void) { return g_last_error.c_str(); }

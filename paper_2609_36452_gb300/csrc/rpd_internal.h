@@ -92,6 +92,9 @@ struct ScoreParams {
     float budget[kMaxBatch];
 };
 
+// Record the message returned by rpd_last_error() on this host thread.
+void set_last_error(const char *msg);
+
 cudaError_t launch_compact(const CompactParams &p, cudaStream_t s);
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s);
 cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, const HeadParams &p,
