@@ -33,6 +33,24 @@ import torch  # noqa: E402
 METRIC = "RPD commit steps/s & rows/s at LLaDA-8B head shape; % of bf16 TC/HBM roofline"
 UNIT = "commit-steps/s"
 
+# DRAM bytes (read + write) per k_head_stats launch from ncu captures, keyed by workload and
+# by a hash of the kernel's sources at capture time; any source change makes it null.
+HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
+                "paper_2609_36452_gb300/csrc/rpd_internal.h")
+HEAD_TRAFFIC = {
+    ("llada_first_step", "f33dc638adb8f691"): 1.0484e9,   # profiles/k_head_stats_llada_first_step.md
+    ("llada_tail_5_masked", "f33dc638adb8f691"): 1.0441e9,  # profiles/k_head_stats_llada_tail5.md
+}
+
+
+def head_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for rel in HEAD_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
 
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -340,6 +358,9 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
         roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": None, "peak_kind": f"HBM copy, of {peaks['source']}"}
     step_roof = max(t_tc, t_hbm) / (ms_step * 1e-3)
+    roof["traffic"] = HEAD_TRAFFIC.get((case["name"], head_source_hash()))
+    roof["algorithmic_bytes"] = bytes_
+    roof["algorithmic_flops"] = flops
 
     cpu = None
     if not args.no_cpu_baseline and world >= 1:
@@ -367,12 +388,89 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
     print(json.dumps(out))
 
 
+def run_trajectory(args):
+    """Decode trajectory at the LLaDA-8B head shape: up to 64 steps on one 256-position
+    canvas; before each step the hidden states are regenerated from the seed for the current
+    mask (context resolves left to right), the step's commits feed the next mask, and the run
+    stops once at most 2% of the canvas is masked.  Each step is timed on the device with
+    CUDA events around the rpd_step call; the per-step roofline time is
+    max(FLOPs / tensor peak, bytes / HBM peak) for that step's masked rows."""
+    import paper_2609_36452_gb300 as rpd
+    import workloads as WL
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    K, N, d, V = 4, 256, WL.LLADA_D, WL.LLADA_V
+    W, g = WL.make_head(V, d, seed=4)
+    Wd, gd = W.to(dev), g.to(dev)
+    gen = torch.Generator().manual_seed(4004)
+    targets = torch.randint(0, V, (N,), generator=gen)
+    ctx = rpd.Rpd(d, V, K, 1e-6)
+    ctx.set_head(Wd, gd)
+    ctx.set_profile("llada")
+    stream = torch.cuda.current_stream(dev)
+    ctx.set_stream(stream)
+    ctx.reserve(1, N)
+    peaks = load_peaks()
+    hidden_d = torch.empty(K, N, d, dtype=torch.bfloat16, device=dev)
+    mask_d = torch.empty(N, dtype=torch.uint8, device=dev)
+    commit = torch.zeros(N, dtype=torch.uint8, device=dev)
+    token = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    stats = torch.zeros(8, dtype=torch.int32, device=dev)
+
+    def trajectory(record):
+        mask = torch.ones(N, dtype=torch.uint8)
+        steps = []
+        for t in range(64):
+            cv = WL.trajectory_hidden(W, K, N, seed=4, step=t, mask=mask, targets=targets)
+            hidden_d.copy_(cv.hidden)
+            mask_d.copy_(mask)
+            torch.cuda.synchronize(dev)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            ctx.step(hidden_d, mask_d, 0.9, 1.0, commit, token, stats)
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            nm = int(mask.sum())
+            st = rpd.stats_dict(stats.cpu())
+            assert st["status"] == 0 and st["n_masked"] == nm, st
+            ms = e0.elapsed_time(e1)
+            R = K * nm
+            roof_s = max(2.0 * R * d * V / (peaks["bf16_tflops"] * 1e12),
+                         (2.0 * V * d + 2.0 * R * d) / (peaks["hbm_gbs"] * 1e9))
+            steps.append({"t": t, "masked": nm, "committed": st["n_committed"], "ms": ms,
+                          "roofline_ms": roof_s * 1e3})
+            mask = mask_d.cpu()
+            if int(mask.sum()) <= 0.02 * N:
+                break
+        return steps
+
+    for _ in range(max(1, args.warmup // 10)):
+        trajectory(False)
+    ctx.profile(True)
+    steps = trajectory(True)
+    ctx.profile(False)
+    kt = ctx.kernel_times(reset=True)
+    total_ms = sum(s["ms"] for s in steps)
+    roof_ms = sum(s["roofline_ms"] for s in steps)
+    out = {
+        "metric": METRIC, "workload": "llada_trajectory", "value": len(steps) / (total_ms / 1e3),
+        "unit": UNIT, "n_gpus": 1, "steps": len(steps), "total_ms": total_ms,
+        "trajectory_roofline_frac": roof_ms / total_ms, "remaining_masked": steps[-1]["masked"] - steps[-1]["committed"],
+        "kernels_ms_total": {k: v[0] for k, v in kt.items()},
+        "per_step": steps, "peaks": peaks,
+    }
+    print(json.dumps(out))
+    ctx.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["rpd", "reference"], default="rpd")
+    ap.add_argument("--workload", choices=["llada_first_step", "trajectory"], default="llada_first_step")
     ap.add_argument("--cpu-positions", type=int, default=32)
     ap.add_argument("--ref-positions", type=int, default=8)
     ap.add_argument("--ref-seconds", type=float, default=150.0)
@@ -385,6 +483,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "trajectory":
+        run_trajectory(args)
     else:
         run_rpd(args)
 
