@@ -9,6 +9,7 @@
 // k_gather_norm (grid-stride, one warp per row): row r = k*NMT + q reads hidden[k][pos(q)],
 //   writes the head operand u[r] = bf16_rne(g * h) (exact product, one rounding) and
 //   inv_rms[r] = (mean(h^2) + eps)^(-1/2); the RMS factor is applied after the contraction.
+#include "ptx.cuh"
 #include "rpd_internal.h"
 
 namespace rpd {
@@ -30,6 +31,8 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
     __shared__ int warp_sum[32];
     __shared__ unsigned long long best_split;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    pdl_wait();
+    pdl_trigger();
     const int total = p.B * p.N;
     int carry = 0;
     for (int base = 0; base < total; base += kCompactThreads * kCompactItems) {
@@ -70,68 +73,118 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
         __syncthreads();
     }
 
-    // Vocabulary split count G for the head kernel: units (m-tile, split) are dealt to the
-    // grid round-robin; minimise waves * n-tiles-per-unit, smallest G on ties.
+    // Head tiling for this step, chosen from the live row count R = K * NMT (no host
+    // round-trip).  For each tiling (single-CTA tiles of 128 rows on `single_slots` CTAs, or
+    // CTA-pair tiles of 256 rows on `pair_slots` pairs) pick the vocabulary split count G
+    // minimising waves * n-tiles-per-unit (smallest G on ties); estimate the time as the
+    // larger of the MMA work of the busiest slot and the head streaming time (scaled by the
+    // vocabulary share of the largest split), in single-tile units; keep the cheaper one.
     const long long nm_rows = static_cast<long long>(p.K) * carry;
-    const long long num_m = (nm_rows + kTileM - 1) / kTileM;
-    if (tid == 0) best_split = ~0ull;
-    __syncthreads();
     const int gmax = min(p.num_n_tiles, p.max_splits);
-    unsigned long long mine = ~0ull;
-    if (num_m > 0) {
+    unsigned long long key1 = ~0ull, key2 = ~0ull;
+    const long long m1 = (nm_rows + kTileM - 1) / kTileM;
+    const long long m2 = (nm_rows + kPairTileM - 1) / kPairTileM;
+    if (tid == 0) best_split = ~0ull;
+    __shared__ unsigned long long best_pair;
+    if (tid == 0) best_pair = ~0ull;
+    __syncthreads();
+    if (m1 > 0) {
         for (int g = tid + 1; g <= gmax; g += kCompactThreads) {
-            const long long units = num_m * g;
-            const long long waves = (units + p.grid_ctas - 1) / p.grid_ctas;
             const long long per = (p.num_n_tiles + g - 1) / g;
-            const unsigned long long key =
-                (static_cast<unsigned long long>(waves * per) << 20) | static_cast<unsigned>(g);
-            mine = key < mine ? key : mine;
+            const long long w1 = (m1 * g + p.single_slots - 1) / p.single_slots;
+            const unsigned long long k1 = (static_cast<unsigned long long>(w1 * per) << 20) | g;
+            key1 = k1 < key1 ? k1 : key1;
+            if (p.pair_slots > 0) {
+                const long long w2 = (m2 * g + p.pair_slots - 1) / p.pair_slots;
+                const unsigned long long k2 = (static_cast<unsigned long long>(w2 * per) << 20) | g;
+                key2 = k2 < key2 ? k2 : key2;
+            }
         }
-        atomicMin(&best_split, mine);
+        atomicMin(&best_split, key1);
+        atomicMin(&best_pair, key2);
     }
     __syncthreads();
     if (tid == 0) {
+        int mode = 1, splits = 1;
+        if (m1 > 0) {
+            const int g1 = static_cast<int>(best_split & 0xFFFFFull);
+            const float per1 = static_cast<float>((p.num_n_tiles + g1 - 1) / g1);
+            const float est1 = fmaxf(static_cast<float>(best_split >> 20),
+                                     p.hbm_tiles * per1 * g1 / p.num_n_tiles);
+            splits = g1;
+            if (p.pair_slots > 0 && best_pair != ~0ull) {
+                const int g2 = static_cast<int>(best_pair & 0xFFFFFull);
+                const float per2 = static_cast<float>((p.num_n_tiles + g2 - 1) / g2);
+                const float est2 = fmaxf(kPairTileCost * static_cast<float>(best_pair >> 20),
+                                         p.hbm_tiles * per2 * g2 / p.num_n_tiles);
+                if (est2 < est1) {
+                    mode = 2;
+                    splits = g2;
+                }
+            }
+        }
         p.canvas_off[p.B] = carry;
         p.meta[kMetaMasked] = carry;
         p.meta[kMetaRows] = static_cast<int>(nm_rows);
         p.meta[kMetaStatus] = RPD_OK;
-        p.meta[kMetaSplits] = num_m > 0 ? static_cast<int>(best_split & 0xFFFFFull) : 1;
+        p.meta[kMetaSplits] = splits;
+        p.meta[kMetaHeadMode] = mode;
     }
 }
 
-__global__ void __launch_bounds__(256) k_gather_norm(NormParams p) {
-    const int nmt = p.meta[kMetaMasked];
-    const int rows = p.meta[kMetaRows];
+// One warp per row; the gain is staged once per CTA in shared memory and each lane keeps up
+// to kVecPerLane 16-byte loads of its row in flight before using any of them.
+constexpr int kNormThreads = 256;
+constexpr int kVecPerLane = 16;  // 32 lanes x 16 x 8 bf16 = 4096 elements per pass
+
+__global__ void __launch_bounds__(kNormThreads) k_gather_norm(NormParams p) {
+    extern __shared__ uint4 g_smem[];
     const int lane = threadIdx.x & 31;
     const int warps_per_cta = blockDim.x >> 5;
     const int nvec = p.d >> 3;  // 8 bf16 per 16-byte vector
-    const uint4 *gvec = reinterpret_cast<const uint4 *>(p.gain);
+    const uint4 *__restrict__ gvec = reinterpret_cast<const uint4 *>(p.gain);
+    for (int v = threadIdx.x; v < nvec; v += blockDim.x) g_smem[v] = __ldg(gvec + v);
+    pdl_wait();
+    pdl_trigger();
+    __syncthreads();
+    const int nmt = p.meta[kMetaMasked];
+    const int rows = p.meta[kMetaRows];
     for (int r = blockIdx.x * warps_per_cta + (threadIdx.x >> 5); r < rows;
          r += gridDim.x * warps_per_cta) {
         const int k = r / nmt;
         const int q = r - k * nmt;
         const int pos = p.pos_of_q[q];
-        const uint4 *src =
+        const uint4 *__restrict__ src =
             reinterpret_cast<const uint4 *>(p.hidden + (static_cast<size_t>(k) * p.BN + pos) * p.d);
-        uint4 *dst = reinterpret_cast<uint4 *>(p.u + static_cast<size_t>(r) * p.d);
+        uint4 *__restrict__ dst = reinterpret_cast<uint4 *>(p.u + static_cast<size_t>(r) * p.d);
         float ss = 0.f;
-        for (int v = lane; v < nvec; v += 32) {
-            const uint4 hv = __ldcs(src + v);
-            const uint4 gv = __ldg(gvec + v);
-            const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&hv);
-            const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gv);
-            uint4 out;
-            __nv_bfloat162 *o2 = reinterpret_cast<__nv_bfloat162 *>(&out);
+        for (int v0 = lane; v0 < nvec; v0 += 32 * kVecPerLane) {
+            uint4 hv[kVecPerLane];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float2 h = __bfloat1622float2(h2[j]);
-                const float2 g = __bfloat1622float2(g2[j]);
-                ss = fmaf(h.x, h.x, ss);
-                ss = fmaf(h.y, h.y, ss);
-                // g*h of two bf16 values is exact in fp32; one RNE to bf16 (reading D1)
-                o2[j] = __float22bfloat162_rn(make_float2(g.x * h.x, g.y * h.y));
+            for (int j = 0; j < kVecPerLane; ++j) {
+                const int v = v0 + 32 * j;
+                if (v < nvec) hv[j] = __ldcs(src + v);
             }
-            dst[v] = out;
+#pragma unroll
+            for (int j = 0; j < kVecPerLane; ++j) {
+                const int v = v0 + 32 * j;
+                if (v >= nvec) break;
+                const uint4 gv = g_smem[v];
+                const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&hv[j]);
+                const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gv);
+                uint4 out;
+                __nv_bfloat162 *o2 = reinterpret_cast<__nv_bfloat162 *>(&out);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 h = __bfloat1622float2(h2[e]);
+                    const float2 g = __bfloat1622float2(g2[e]);
+                    ss = fmaf(h.x, h.x, ss);
+                    ss = fmaf(h.y, h.y, ss);
+                    // g*h of two bf16 values is exact in fp32; one RNE to bf16 (reading D1)
+                    o2[e] = __float22bfloat162_rn(make_float2(g.x * h.x, g.y * h.y));
+                }
+                dst[v] = out;
+            }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
@@ -142,13 +195,17 @@ __global__ void __launch_bounds__(256) k_gather_norm(NormParams p) {
 }  // namespace
 
 cudaError_t launch_compact(const CompactParams &p, cudaStream_t s) {
-    k_compact<<<1, kCompactThreads, 0, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(k_compact, dim3(1), dim3(kCompactThreads), 0, s, p);
 }
 
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s) {
-    k_gather_norm<<<grid, 256, 0, s>>>(p);
-    return cudaGetLastError();
+    const size_t smem = static_cast<size_t>(p.d) * 2;  // the gain, staged once per CTA
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(k_gather_norm, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+    }
+    return launch_pdl(k_gather_norm, dim3(grid), dim3(kNormThreads), smem, s, p);
 }
 
 }  // namespace rpd

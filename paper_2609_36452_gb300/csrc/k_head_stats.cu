@@ -80,6 +80,8 @@ __device__ __forceinline__ void fold_chunk(const float (&v)[32], float scale, in
 __global__ void __launch_bounds__(kHeadThreads, 1)
     k_head_stats(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW,
                  HeadParams p) {
+    pdl_wait();  // row count, tiling, u and inv_rms come from the preceding kernels
+    if (p.meta[kMetaHeadMode] != 1) return;  // the CTA-pair tiling runs this step
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -96,14 +98,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-
-    const int rows = p.meta[kMetaRows];
-    TileWalk tw;
-    tw.num_m = (rows + kTileM - 1) / kTileM;
-    tw.num_n = (p.V + kTileN - 1) / kTileN;
-    tw.splits = p.meta[kMetaSplits];
-    tw.units = tw.num_m * tw.splits;
-    const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kStages; ++i) {
@@ -125,6 +119,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     __syncthreads();
     tc_fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
+
+    const int rows = p.meta[kMetaRows];
+    TileWalk tw;
+    tw.num_m = (rows + kTileM - 1) / kTileM;
+    tw.num_n = (p.V + kTileN - 1) / kTileN;
+    tw.splits = p.meta[kMetaSplits];
+    tw.units = tw.num_m * tw.splits;
+    const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -259,6 +261,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     }
 
     __syncwarp();
+    pdl_trigger();  // the merge kernel may launch once every CTA is past its main loop
     tc_fence_before_sync();
     __syncthreads();
     tc_fence_after_sync();
@@ -266,6 +269,227 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     if (warp == 1) {
         __syncwarp();
         tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+
+// ------------------------------------------------------------------------------------------
+// CTA-pair form (tcgen05 cta_group::2).  A pair (cluster of 2 CTAs) computes a tile of 256
+// rows x 256 vocabulary columns: CTA r of the pair stages rows [128r, 128r+128) of the row
+// tile and W rows [128r, 128r+128) of the vocabulary tile; the even CTA issues
+// tcgen05.mma.cta_group::2 with M=256, N=256, which reads both CTAs' shared memory and
+// accumulates rows [128r, 128r+128) x all 256 columns into CTA r's TMEM.  Per SM and K-step
+// that is 32 KB of operands for the same MMA work the single-CTA tile does with 48 KB.
+//
+// Barriers: full[s] lives in the even CTA and receives both CTAs' TMA completions (tx bytes
+// 64 KB per stage); empty[s], acc_full[a] and drain receive multicast commits from the MMA
+// thread in both CTAs; acc_empty[a] lives in the even CTA and counts the 4 epilogue warps
+// of both CTAs (8 arrivals).
+__global__ void __launch_bounds__(kHeadThreads, 1)
+    k_head_stats_pair(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW,
+                      HeadParams p) {
+    pdl_wait();  // row count, tiling, u and inv_rms come from the preceding kernels
+    if (p.meta[kMetaHeadMode] != 2) return;  // the single-CTA tiling runs this step
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + kPairStages * kPairStageBytesA;
+    uint64_t *bars =
+        reinterpret_cast<uint64_t *>(smem + kPairStages * (kPairStageBytesA + kPairStageBytesB));
+    uint64_t *full = bars;                            // [kPairStages] (used in the even CTA)
+    uint64_t *empty = bars + kPairStages;             // [kPairStages]
+    uint64_t *acc_full = bars + 2 * kPairStages;      // [2]
+    uint64_t *acc_empty = bars + 2 * kPairStages + 2; // [2] (used in the even CTA)
+    uint64_t *drain = bars + 2 * kPairStages + 4;     // [1]
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kPairStages + 5);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();  // 0 = even CTA (issues the MMAs), 1 = odd
+    const int pair = blockIdx.x >> 1;
+    const int num_pairs = gridDim.x >> 1;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kPairStages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_empty[i], 8);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tma_prefetch_desc(&tmU);
+        tma_prefetch_desc(&tmW);
+    }
+    if (warp == 1) tmem_alloc_pair(tmem_slot, kTmemCols);
+    tc_fence_before_sync();
+    __syncthreads();
+    cluster_sync();  // both CTAs' barriers initialised before any cross-CTA signal
+    tc_fence_after_sync();
+    const uint32_t tmem_base = *tmem_slot;
+
+    const int rows = p.meta[kMetaRows];
+    TileWalk tw;
+    tw.num_m = (rows + kPairTileM - 1) / kPairTileM;
+    tw.num_n = (p.V + kTileN - 1) / kTileN;
+    tw.splits = p.meta[kMetaSplits];
+    tw.units = tw.num_m * tw.splits;
+    const int num_kb = (p.d + kTileK - 1) / kTileK;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ------------------------------------------------------- TMA producer (both CTAs)
+            const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);
+            int stage = 0;
+            uint32_t phase = 0;
+            long long fills = 0;
+            bool ok = true;
+            for (int u = pair; ok && u < tw.units; u += num_pairs) {
+                int m, n0, n1;
+                tw.unit(u, m, n0, n1);
+                for (int n = n0; ok && n < n1; ++n) {
+                    for (int kb = 0; kb < num_kb; ++kb) {
+                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
+                            ok = false;
+                            break;
+                        }
+                        if (rank == 0)
+                            mbar_arrive_expect_tx(&full[stage], 2 * (kPairStageBytesA + kPairStageBytesB));
+                        const uint32_t fb = full0 + static_cast<uint32_t>(stage * sizeof(uint64_t));
+                        tma_load_2d_pair(sA + stage * kPairStageBytesA, &tmU, fb, kb * kTileK,
+                                         m * kPairTileM + static_cast<int>(rank) * kPairHalfRows);
+                        tma_load_2d_pair(sB + stage * kPairStageBytesB, &tmW, fb, kb * kTileK,
+                                         n * kTileN + static_cast<int>(rank) * kPairHalfRows);
+                        ++fills;
+                        if (++stage == kPairStages) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                    }
+                }
+            }
+            // Drain: a stage's copy has landed once the MMAs that read it have completed, which
+            // the multicast commit on empty[s] reports in this CTA.
+            for (int s = 0; s < kPairStages; ++s) {
+                const long long n_s = fills / kPairStages + (s < fills % kPairStages ? 1 : 0);
+                if (n_s > 0)
+                    mbar_wait_drain(&empty[s], static_cast<uint32_t>((n_s - 1) & 1), kWaitLimitNs / 8);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            if (rank == 0) {
+                // ------------------------------------------------ MMA issuer (even CTA only)
+                constexpr uint32_t idesc = idesc_bf16_f32(kPairTileM, kTileN);
+                int stage = 0;
+                uint32_t phase = 0;
+                uint32_t tile_iter = 0;
+                bool ok = true;
+                for (int u = pair; ok && u < tw.units; u += num_pairs) {
+                    int m, n0, n1;
+                    tw.unit(u, m, n0, n1);
+                    for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
+                        const uint32_t acc = tile_iter & 1u;
+                        const uint32_t acc_phase = (tile_iter >> 1) & 1u;
+                        if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
+                                               kWaitLimitNs)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after_sync();
+                        const uint32_t d_tmem = tmem_base + acc * kTileN;
+                        for (int kb = 0; kb < num_kb; ++kb) {
+                            if (!mbar_wait_bounded(&full[stage], phase, abort_flag, kWaitLimitNs)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after_sync();
+                            const uint32_t a0 = smem_u32(sA + stage * kPairStageBytesA);
+                            const uint32_t b0 = smem_u32(sB + stage * kPairStageBytesB);
+#pragma unroll
+                            for (int kk = 0; kk < kTileK / 16; ++kk) {
+                                umma_bf16_pair(d_tmem, smem_desc_sw128(a0 + kk * 32),
+                                               smem_desc_sw128(b0 + kk * 32), idesc,
+                                               (kb > 0 || kk > 0) ? 1u : 0u);
+                            }
+                            umma_commit_pair_multicast(&empty[stage], 0x3);
+                            if (++stage == kPairStages) {
+                                stage = 0;
+                                phase ^= 1u;
+                            }
+                        }
+                        if (!ok) break;
+                        umma_commit_pair_multicast(&acc_full[acc], 0x3);
+                    }
+                }
+                umma_commit_pair_multicast(drain, 0x3);
+            }
+            // Both CTAs: every MMA writing this CTA's TMEM has completed before it is freed.
+            mbar_wait_drain(drain, 0, kWaitLimitNs);
+        }
+    } else {
+        // ---------------------------------------------------------- epilogue (both CTAs)
+        const int sub = warp & 3;
+        const int row_in_tile = static_cast<int>(rank) * kPairHalfRows + sub * 32 + lane;
+        const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
+        const uint32_t acc_empty0 = mapa_shared(smem_u32(&acc_empty[0]), 0);
+        uint32_t tile_iter = 0;
+        bool ok = true;
+        for (int u = pair; ok && u < tw.units; u += num_pairs) {
+            int m, n0, n1;
+            tw.unit(u, m, n0, n1);
+            const int r = m * kPairTileM + row_in_tile;
+            const bool valid = r < rows;
+            const float scale = valid ? p.inv_rms[r] * kLog2e : 0.f;
+            float run_m = -INFINITY, run_s = 0.f, run_t = 0.f;
+            int run_a = 0;
+            for (int n = n0; n < n1; ++n, ++tile_iter) {
+                const uint32_t acc = tile_iter & 1u;
+                const uint32_t acc_phase = (tile_iter >> 1) & 1u;
+                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, kWaitLimitNs)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after_sync();
+                const int col_base = n * kTileN;
+                const bool full_tile = col_base + kTileN <= p.V;
+#pragma unroll 1
+                for (int c = 0; c < kTileN / 32; ++c) {
+                    float v[32];
+                    tmem_ld_32x32b_x32(lane_base + acc * kTileN + c * 32, v);
+                    if (full_tile)
+                        fold_chunk<true>(v, scale, col_base + c * 32, p.V, run_m, run_s, run_t, run_a);
+                    else
+                        fold_chunk<false>(v, scale, col_base + c * 32, p.V, run_m, run_s, run_t, run_a);
+                }
+                tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(acc_empty0 + acc * static_cast<uint32_t>(sizeof(uint64_t)));
+            }
+            if (!ok) break;
+            if (valid) {
+                const int g = u / tw.num_m;
+                p.partials[static_cast<size_t>(r) * p.max_splits + g] =
+                    make_float4(run_m, run_s, run_t, __int_as_float(run_a));
+            }
+        }
+    }
+
+    __syncwarp();
+    pdl_trigger();
+    tc_fence_before_sync();
+    __syncthreads();
+    cluster_sync();  // no signal may still be in flight to a CTA that is about to exit
+    tc_fence_after_sync();
+    if (*abort_flag && threadIdx.x == 0) atomicExch(&p.meta[kMetaStatus], RPD_ERR_TIMEOUT);
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc_pair(tmem_base, kTmemCols);
     }
 }
 
@@ -280,8 +504,60 @@ cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, co
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    k_head_stats<<<grid, kHeadThreads, kHeadSmemBytes, s>>>(tmU, tmW, p);
-    return cudaGetLastError();
+    return launch_pdl(k_head_stats, dim3(grid), dim3(kHeadThreads), kHeadSmemBytes, s, tmU, tmW, p);
+}
+
+}  // namespace rpd
+
+namespace rpd {
+
+int head_stats_pair_max_clusters() {
+    static int cached = -1;
+    if (cached >= 0) return cached;
+    cudaError_t e = cudaFuncSetAttribute(k_head_stats_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kPairSmemBytes);
+    if (e != cudaSuccess) return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2);
+    cfg.blockDim = dim3(kHeadThreads);
+    cfg.dynamicSmemBytes = kPairSmemBytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k_head_stats_pair, &cfg) != cudaSuccess) n = 0;
+    cached = n;
+    return n;
+}
+
+cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tmW,
+                                   const HeadParams &p, int grid, cudaStream_t s) {
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(k_head_stats_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kPairSmemBytes);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kHeadThreads);
+    cfg.dynamicSmemBytes = kPairSmemBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, k_head_stats_pair, tmU, tmW, p);
 }
 
 }  // namespace rpd

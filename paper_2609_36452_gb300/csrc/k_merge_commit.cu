@@ -23,6 +23,7 @@
 //   If nothing is accepted and something is masked, commit the most confident of the
 //   first W masked positions (leftmost on ties, §3.2).  Then write the outputs, clear the
 //   committed mask bits and the per-canvas counters.
+#include "ptx.cuh"
 #include "rpd_internal.h"
 
 namespace rpd {
@@ -49,6 +50,8 @@ __device__ __forceinline__ Stat merge2(const Stat &x, const Stat &y) {
 }
 
 __global__ void __launch_bounds__(256) k_merge(MergeParams p) {
+    pdl_wait();
+    pdl_trigger();
     const int rows = p.meta[kMetaRows];
     const int splits = p.meta[kMetaSplits];
     const int lane = threadIdx.x & 31;
@@ -80,50 +83,80 @@ __global__ void __launch_bounds__(256) k_merge(MergeParams p) {
 
 // ------------------------------------------------------------------ block-wide helpers
 
-template <typename T>
-__device__ __forceinline__ T warp_incl_scan(T v, int lane) {
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const T t = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= o) v += t;
-    }
-    return v;
-}
+struct ScanPair {
+    float q;  // entropy of masked non-candidates
+    int m;    // masked positions
+};
 
-// Exclusive scan over the block in thread order; `sh` holds 32 entries.
-template <typename T>
-__device__ __forceinline__ T block_excl_scan(T v, T *sh, T &total) {
+// Exclusive scan of (q, m) in thread order over the block, plus the block totals.
+__device__ __forceinline__ ScanPair block_scan_pair(ScanPair v, ScanPair *sh, ScanPair &total) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nwarps = (blockDim.x + 31) >> 5;
-    const T incl = warp_incl_scan(v, lane);
-    __syncthreads();
+    ScanPair incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float tq = __shfl_up_sync(0xffffffffu, incl.q, o);
+        const int tm = __shfl_up_sync(0xffffffffu, incl.m, o);
+        if (lane >= o) {
+            incl.q += tq;
+            incl.m += tm;
+        }
+    }
     if (lane == 31) sh[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-        const T w = lane < nwarps ? sh[lane] : T(0);
-        const T wi = warp_incl_scan(w, lane);
-        sh[lane] = wi - w;
+        ScanPair w = lane < nwarps ? sh[lane] : ScanPair{0.f, 0};
+        ScanPair wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float tq = __shfl_up_sync(0xffffffffu, wi.q, o);
+            const int tm = __shfl_up_sync(0xffffffffu, wi.m, o);
+            if (lane >= o) {
+                wi.q += tq;
+                wi.m += tm;
+            }
+        }
+        sh[lane] = ScanPair{wi.q - w.q, wi.m - w.m};
         if (lane == 31) sh[32] = wi;
     }
     __syncthreads();
     total = sh[32];
-    return sh[warp] + incl - v;
+    const ScanPair base = sh[warp];
+    return ScanPair{base.q + incl.q - v.q, base.m + incl.m - v.m};
 }
 
-template <typename T>
-__device__ __forceinline__ T block_sum(T v, T *sh) {
-    T total;
-    block_excl_scan(v, sh, total);
-    return total;
+// Block-wide sums of three counters.
+__device__ __forceinline__ int3 block_sum3(int3 v, int3 *sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nwarps = (blockDim.x + 31) >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        v.x += __shfl_xor_sync(0xffffffffu, v.x, o);
+        v.y += __shfl_xor_sync(0xffffffffu, v.y, o);
+        v.z += __shfl_xor_sync(0xffffffffu, v.z, o);
+    }
+    if (lane == 0) sh[warp] = v;
+    __syncthreads();
+    int3 t = make_int3(0, 0, 0);
+    for (int w = 0; w < nwarps; ++w) {
+        t.x += sh[w].x;
+        t.y += sh[w].y;
+        t.z += sh[w].z;
+    }
+    return t;
 }
+
+constexpr int kLayerBatch = 8;  // window layers whose statistics are loaded together
 
 __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p) {
     constexpr int kMaxItems = kMaxCanvas / kScoreThreads;
-    __shared__ float shf[33];
-    __shared__ int shi[33];
+    __shared__ ScanPair sh_scan[33];
+    __shared__ int3 sh_sum[32];
     __shared__ int first_reject;
     __shared__ unsigned long long best_fb;
 
+    pdl_wait();
+    pdl_trigger();
     const int b = blockIdx.x;
     const int N = p.N;
     const int nmt = p.meta[kMetaMasked];
@@ -132,13 +165,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     const int items = (N + blockDim.x - 1) / blockDim.x;
     const int i0 = threadIdx.x * items;
     uint8_t *mask = p.mask + static_cast<size_t>(b) * N;
+    const bool dbg_layers = p.dbg.layer_argmax || p.dbg.layer_pmax;
 
     bool masked[kMaxItems], cand[kMaxItems], high[kMaxItems];
     int y[kMaxItems];
     float conf[kMaxItems], H[kMaxItems];
 
-    int n_masked = 0, n_cand = 0;
-    float local_q = 0.f;
+    ScanPair local{0.f, 0};
+    int n_cand = 0;
 #pragma unroll
     for (int j = 0; j < kMaxItems; ++j) {
         masked[j] = cand[j] = high[j] = false;
@@ -152,34 +186,55 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
         float r = 0.f, s = 0.f;
         if (masked[j]) {
             const int q = p.q_of_pos[pos];
-            const size_t last = static_cast<size_t>(K - 1) * nmt + q;
-            y[j] = p.row_arg[last];
-            conf[j] = p.row_pmax[last];
-            H[j] = p.row_H[last];
-            ki = 1;
-            float peak = conf[j];
-            for (int k = K - 2; k >= 0; --k) {
-                const size_t rk = static_cast<size_t>(k) * nmt + q;
-                if (p.row_arg[rk] != y[j]) break;
-                ++ki;
-                peak = fmaxf(peak, p.row_pmax[rk]);
+            // Backward over the window, a batch of layers at a time (loads issued together).
+            float peak = 0.f;
+            bool run = true;
+            for (int k_hi = K; k_hi > 0; k_hi -= kLayerBatch) {
+                if (!run && !dbg_layers) break;  // persistence settled; debug wants every layer
+                int a_b[kLayerBatch];
+                float p_b[kLayerBatch];
+#pragma unroll
+                for (int t = 0; t < kLayerBatch; ++t) {
+                    const int k = k_hi - 1 - t;
+                    if (k >= 0) {
+                        const size_t rk = static_cast<size_t>(k) * nmt + q;
+                        a_b[t] = p.row_arg[rk];
+                        p_b[t] = p.row_pmax[rk];
+                    }
+                }
+#pragma unroll
+                for (int t = 0; t < kLayerBatch; ++t) {
+                    const int k = k_hi - 1 - t;
+                    if (k < 0) break;
+                    if (k == K - 1) {
+                        y[j] = a_b[t];
+                        conf[j] = p_b[t];
+                        peak = p_b[t];
+                        ki = 1;
+                    } else if (run) {
+                        if (a_b[t] != y[j]) {
+                            run = false;
+                        } else {
+                            ++ki;
+                            peak = fmaxf(peak, p_b[t]);
+                        }
+                    }
+                    if (dbg_layers) {
+                        const size_t o = (static_cast<size_t>(k) * p.B) * N + pos;
+                        if (p.dbg.layer_argmax) p.dbg.layer_argmax[o] = a_b[t];
+                        if (p.dbg.layer_pmax) p.dbg.layer_pmax[o] = p_b[t];
+                    }
+                }
             }
+            H[j] = p.row_H[static_cast<size_t>(K - 1) * nmt + q];
             r = peak - conf[j];
             s = static_cast<float>(min(ki, p.k_max)) - p.w * r;
             high[j] = conf[j] >= tau;
             cand[j] = high[j] || (conf[j] >= p.theta_c && conf[j] < tau && s >= p.theta_s);
-            ++n_masked;
+            ++local.m;
             n_cand += cand[j];
-            if (!cand[j]) local_q += H[j];
-            if (p.dbg.layer_argmax || p.dbg.layer_pmax) {
-                for (int k = 0; k < K; ++k) {
-                    const size_t rk = static_cast<size_t>(k) * nmt + q;
-                    const size_t o = (static_cast<size_t>(k) * p.B) * N + pos;
-                    if (p.dbg.layer_argmax) p.dbg.layer_argmax[o] = p.row_arg[rk];
-                    if (p.dbg.layer_pmax) p.dbg.layer_pmax[o] = p.row_pmax[rk];
-                }
-            }
-        } else if (p.dbg.layer_argmax || p.dbg.layer_pmax) {
+            if (!cand[j]) local.q += H[j];
+        } else if (dbg_layers) {
             for (int k = 0; k < K; ++k) {
                 const size_t o = (static_cast<size_t>(k) * p.B) * N + pos;
                 if (p.dbg.layer_argmax) p.dbg.layer_argmax[o] = -1;
@@ -194,11 +249,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
         if (p.dbg.candidate) p.dbg.candidate[pos] = cand[j];
     }
 
-    // ------------------------------------------- entropy of masked non-candidates, scanned
-    float q_total;
-    float q = block_excl_scan(local_q, shf, q_total);
-    if (threadIdx.x == 0) first_reject = N;
-    __syncthreads();
+    // ------------------------------ entropy of masked non-candidates and masked ranks, scanned
+    if (threadIdx.x == 0) {
+        first_reject = N;
+        best_fb = 0ull;
+    }
+    ScanPair total;
+    const ScanPair pre = block_scan_pair(local, sh_scan, total);  // synchronises the block
+    float q = pre.q;
 #pragma unroll
     for (int j = 0; j < kMaxItems; ++j) {
         if (j >= items || i0 + j >= N) break;
@@ -211,25 +269,20 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     __syncthreads();
     const int reject_at = first_reject;
 
-    int n_acc = 0, n_high = 0;
+    int3 cnt = make_int3(0, 0, n_cand);  // accepted, accepted through c >= tau, candidates
 #pragma unroll
     for (int j = 0; j < kMaxItems; ++j) {
         const bool acc = cand[j] && (i0 + j) < reject_at;
-        n_acc += acc;
-        n_high += acc && high[j];
+        cnt.x += acc;
+        cnt.y += acc && high[j];
     }
-    int dummy;
-    const int total_masked = block_sum(n_masked, shi);
-    const int total_acc = block_sum(n_acc, shi);
-    const int total_cand = block_sum(n_cand, shi);
-    const int total_high = block_sum(n_high, shi);
+    const int3 tot = block_sum3(cnt, sh_sum);
+    const int total_masked = total.m;
 
     // ------------------------------------------------------------------------ fallback
     int fb_pos = -1;
-    if (total_acc == 0 && total_masked > 0) {
-        int rank = block_excl_scan(n_masked, shi, dummy);
-        if (threadIdx.x == 0) best_fb = 0ull;
-        __syncthreads();
+    if (tot.x == 0 && total_masked > 0) {  // uniform across the block
+        int rank = pre.m;
         unsigned long long mine = 0ull;
 #pragma unroll
         for (int j = 0; j < kMaxItems; ++j) {
@@ -264,10 +317,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     if (threadIdx.x == 0) {
         rpd_stats st;
         st.n_masked = total_masked;
-        st.n_candidates = total_cand;
-        st.n_high_conf = total_high;
-        st.n_stability = total_acc - total_high;
-        st.n_committed = total_acc + (fb_pos >= 0 ? 1 : 0);
+        st.n_candidates = tot.z;
+        st.n_high_conf = tot.y;
+        st.n_stability = tot.x - tot.y;
+        st.n_committed = tot.x + (fb_pos >= 0 ? 1 : 0);
         st.fallback_used = fb_pos >= 0 ? 1 : 0;
         st.fallback_pos = fb_pos;
         st.status = p.meta[kMetaStatus];
@@ -278,14 +331,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
 }  // namespace
 
 cudaError_t launch_merge(const MergeParams &p, int grid, cudaStream_t s) {
-    k_merge<<<grid, 256, 0, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(k_merge, dim3(grid), dim3(256), 0, s, p);
 }
 
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s) {
     const int threads = p.N >= kScoreThreads ? kScoreThreads : ((p.N + 31) / 32) * 32;
-    k_score_commit<<<p.B, threads, 0, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(k_score_commit, dim3(p.B), dim3(threads), 0, s, p);
 }
 
 }  // namespace rpd

@@ -11,6 +11,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -94,7 +95,8 @@ struct rpd_ctx {
     int32_t *row_arg = nullptr;
     float *row_pmax = nullptr, *row_H = nullptr;
     int32_t *q_of_pos = nullptr, *pos_of_q = nullptr, *canvas_off = nullptr, *meta = nullptr;
-    CUtensorMap tmU{}, tmW{};
+    CUtensorMap tmU{}, tmW{}, tmW_pair{};
+    int pair_grid = 0;   // CTAs of the CTA-pair head kernel (2 x resident pairs; 0 = none)
 
     // host-buffer entry point staging
     size_t stage_bytes = 0;
@@ -242,12 +244,13 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
 
     const int bn = B * N;
     const int num_n = (c->V + kTileN - 1) / kTileN;
-    const int grid_head = c->num_sms;
+    const int pair_slots = c->pair_grid / 2;
     cudaError_t e;
     {
         KernelTimer t(c, 0);
         CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
-                         num_n, grid_head, c->max_splits};
+                         num_n, c->max_splits, c->num_sms, pair_slots,
+                         head_stream_in_tiles(c->V, c->d, c->num_sms)};
         e = launch_compact(cp, c->stream);
         if (e == cudaSuccess) {
             NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
@@ -260,7 +263,11 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
     {
         KernelTimer t(c, 1);
         HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits};
-        e = launch_head_stats(c->tmU, c->tmW, hp, grid_head, c->stream);
+        // Both tilings are launched; each reads the choice k_compact made for this step's row
+        // count and the other returns at once.
+        e = launch_head_stats(c->tmU, c->tmW, hp, c->num_sms, c->stream);
+        if (e == cudaSuccess && pair_slots > 0)
+            e = launch_head_stats_pair(c->tmU, c->tmW_pair, hp, c->pair_grid, c->stream);
     }
     if (e != cudaSuccess) return cuda_fail(e, "head statistics launch");
     {
@@ -349,6 +356,8 @@ rpd_ctx *rpd_create(int d, int V, int K, float eps) {
         delete c;
         return nullptr;
     }
+    const int clusters = head_stats_pair_max_clusters();
+    c->pair_grid = 2 * std::min(clusters, c->num_sms / 2);
     return c;
 }
 
@@ -356,10 +365,13 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
     if (!c || !W_head || !g_norm) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
     if (!aligned16(W_head) || !aligned16(g_norm))
         return fail(RPD_ERR_INVALID_ARGUMENT, "W_head and g_norm must be 16-byte aligned");
-    CUtensorMap m;
+    CUtensorMap m, m2;
     int rc = encode_bf16_2d(&m, W_head, static_cast<uint64_t>(c->V), c->d, kTileN);
     if (rc) return rc;
+    rc = encode_bf16_2d(&m2, W_head, static_cast<uint64_t>(c->V), c->d, kPairHalfRows);
+    if (rc) return rc;
     c->tmW = m;
+    c->tmW_pair = m2;
     c->W = W_head;
     c->g = g_norm;
     return RPD_OK;

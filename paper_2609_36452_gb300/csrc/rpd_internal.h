@@ -20,6 +20,14 @@ constexpr int kHeadThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM owner, warps
 constexpr int kStageBytesA = kTileM * kTileK * 2;
 constexpr int kStageBytesB = kTileN * kTileK * 2;
 constexpr int kHeadSmemBytes = kStages * (kStageBytesA + kStageBytesB) + 1024 + 256;
+// CTA-pair variant: a pair computes 256 rows x 256 vocabulary columns per tile; each CTA
+// stages its own 128 rows of u and 128 rows of W per K-step (32 KB), 6 stages deep.
+constexpr int kPairTileM = 256;
+constexpr int kPairStages = 6;
+constexpr int kPairHalfRows = 128;
+constexpr int kPairStageBytesA = kPairHalfRows * kTileK * 2;
+constexpr int kPairStageBytesB = kPairHalfRows * kTileK * 2;
+constexpr int kPairSmemBytes = kPairStages * (kPairStageBytesA + kPairStageBytesB) + 1024 + 256;
 constexpr int kMaxBatch = 128;
 constexpr int kMaxCanvas = 8192;
 constexpr int kScoreThreads = 1024;
@@ -31,6 +39,7 @@ enum MetaIndex : int {
     kMetaRows = 1,     // projected rows R = K * NMT
     kMetaStatus = 2,   // RPD_OK or RPD_ERR_TIMEOUT, latched by kernels
     kMetaSplits = 3,   // vocabulary splits G chosen for the head kernel
+    kMetaHeadMode = 4, // 1: single-CTA head tiles, 2: CTA-pair head tiles
     kMetaWords = 8
 };
 
@@ -42,9 +51,19 @@ struct CompactParams {
     int32_t *meta;        // [kMetaWords]
     int B, N, K;
     int num_n_tiles;      // ceil(V / kTileN)
-    int grid_ctas;        // CTAs of the head kernel
     int max_splits;       // capacity of the partial-statistics buffer per row
+    int single_slots;     // CTAs of the single-CTA head kernel
+    int pair_slots;       // CTA pairs of the pair head kernel (0: pair tiles unavailable)
+    float hbm_tiles;      // time to stream the head once, in single-CTA tile times
 };
+
+// Relative cost of a CTA-pair tile (256 rows on two SMs) against a single-CTA tile (128 rows
+// on one SM): measured per-SM throughput of the pair form on GB300 at the LLaDA head shape.
+constexpr float kPairTileCost = 0.88f;
+// Per-SM rate of the single-CTA tile and the sustained HBM read rate used by the tiling
+// choice (GB300 measurements; only their ratio matters).
+constexpr double kSingleTileFlopsPerSm = 1.1e13;
+constexpr double kHeadStreamBytesPerSec = 6.5e12;
 
 struct NormParams {
     const __nv_bfloat16 *hidden;  // [K][B*N][d]
@@ -63,6 +82,14 @@ struct HeadParams {
     int32_t *meta;
     int V, d, max_splits;
 };
+
+// Time to stream the head once, in units of one single-CTA tile's MMA time.
+inline float head_stream_in_tiles(int V, int d, int num_sms) {
+    (void)num_sms;
+    const double t_hbm = 2.0 * V * static_cast<double>(d) / kHeadStreamBytesPerSec;
+    const double t_tile = 2.0 * kTileM * kTileN * static_cast<double>(d) / kSingleTileFlopsPerSm;
+    return static_cast<float>(t_hbm / t_tile);
+}
 
 struct MergeParams {
     const float4 *partials;
@@ -92,6 +119,25 @@ struct ScoreParams {
     float budget[kMaxBatch];
 };
 
+// Launch with programmatic stream serialisation, so that the kernel's prologue overlaps the
+// tail of its predecessor in the stream (the kernel itself waits with griddepcontrol.wait
+// before it reads what the predecessor wrote).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 // Record the message returned by rpd_last_error() on this host thread.
 void set_last_error(const char *msg);
 
@@ -99,6 +145,11 @@ cudaError_t launch_compact(const CompactParams &p, cudaStream_t s);
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s);
 cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, const HeadParams &p,
                               int grid, cudaStream_t s);
+// tmU/tmW boxes: 64 x 128 rows.  grid = 2 x (pairs); clusters of 2 CTAs.
+cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tmW,
+                                   const HeadParams &p, int grid, cudaStream_t s);
+// Largest number of CTA pairs of the pair kernel that can be resident at once.
+int head_stats_pair_max_clusters();
 cudaError_t launch_merge(const MergeParams &p, int grid, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
 

@@ -27,6 +27,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <mutex>
@@ -65,6 +66,7 @@ struct DeviceSetup {
     bool ready = false;
     uint8_t *arena = nullptr;  // device address of g_noalloc_arena on this device
     int num_sms = 0;
+    int pair_grid = 0;         // CTAs of the CTA-pair head kernel (same choice as rpd_step)
 };
 
 std::mutex g_setup_mutex;
@@ -121,6 +123,7 @@ int setup_device(DeviceSetup **out) {
         if (e != cudaSuccess) return na_fail(RPD_ERR_CUDA, "cudaDeviceGetAttribute failed");
         s.arena = static_cast<uint8_t *>(ptr);
         s.num_sms = sms;
+        s.pair_grid = 2 * std::min(head_stats_pair_max_clusters(), sms / 2);
         s.ready = true;
     }
     *out = &s;
@@ -181,9 +184,13 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     int32_t *canvas_off = reinterpret_cast<int32_t *>(A + kOffCanvasOff);
     int32_t *meta = reinterpret_cast<int32_t *>(A + kOffMeta);
 
-    CUtensorMap tmU, tmW;
+    // Same head-kernel configuration as rpd_step (both tilings, chosen on the device).
+    const int pair_slots = dev->pair_grid / 2;
+    CUtensorMap tmU, tmW, tmW_pair;
     if (!encode_tile_map(&tmU, u, kNaMaxRows, static_cast<uint64_t>(d), kTileM) ||
-        !encode_tile_map(&tmW, W_head, static_cast<uint64_t>(V), static_cast<uint64_t>(d), kTileN))
+        !encode_tile_map(&tmW, W_head, static_cast<uint64_t>(V), static_cast<uint64_t>(d), kTileN) ||
+        !encode_tile_map(&tmW_pair, W_head, static_cast<uint64_t>(V), static_cast<uint64_t>(d),
+                         kPairHalfRows))
         return na_fail(RPD_ERR_CUDA, "cuTensorMapEncodeTiled failed");
 
     const int num_n = (V + kTileN - 1) / kTileN;
@@ -193,8 +200,8 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     // The per-step count/status words must start from zero on every call.
     cudaError_t e = cudaMemsetAsync(meta, 0, kMetaWords * 4, stream);
     if (e == cudaSuccess) {
-        CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n,
-                         dev->num_sms, splits};
+        CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n, splits,
+                         dev->num_sms, pair_slots, head_stream_in_tiles(V, d, dev->num_sms)};
         e = launch_compact(cp, stream);
     }
     if (e == cudaSuccess) {
@@ -206,6 +213,8 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     if (e == cudaSuccess) {
         HeadParams hp{inv_rms, partials, meta, V, d, splits};
         e = launch_head_stats(tmU, tmW, hp, dev->num_sms, stream);
+        if (e == cudaSuccess && pair_slots > 0)
+            e = launch_head_stats_pair(tmU, tmW_pair, hp, dev->pair_grid, stream);
     }
     if (e == cudaSuccess) {
         MergeParams mp{partials, meta, row_arg, row_pmax, row_H, splits};

@@ -40,6 +40,7 @@ def test_masks():
 def test_trajectory_profile_rises_with_committed_prefix():
     base = torch.ones(8)
     mask = torch.tensor([0, 0, 0, 0, 1, 1, 1, 1], dtype=torch.uint8)
-    b = WL.trajectory_profile(base, mask, boost=3.0)
-    assert math.isclose(b[0].item(), 1.0) and math.isclose(b[4].item(), 4.0)
-    assert math.isclose(b[7].item(), 1 + 3 * 4 / 7, rel_tol=1e-6)
+    b = WL.trajectory_profile(base, mask, b_hi=4.0, gamma=2.0)
+    assert math.isclose(b[0].item(), 4.0)                      # nothing to its left
+    assert math.isclose(b[4].item(), 4.0)                      # whole prefix committed
+    assert math.isclose(b[7].item(), 1 + 3 * (4 / 7) ** 2, rel_tol=1e-6)

@@ -229,21 +229,27 @@ def batched_serving(seed: int = 5, kappa: float = DEFAULT_KAPPA, B: int = 8, N: 
                 canvases=canvases, seed=seed, kappa=kappa)
 
 
-def trajectory_profile(base_b: torch.Tensor, mask: torch.Tensor, boost: float = 3.0) -> torch.Tensor:
-    """Signal profile for a decode-trajectory step: ``b_p * (1 + boost * f_p)`` where ``f_p`` is
-    the committed fraction of the positions before p.  Context resolves left to right."""
+def trajectory_profile(base_b: torch.Tensor, mask: torch.Tensor, b_hi: float = 4.0,
+                       gamma: float = 8.0) -> torch.Tensor:
+    """Signal profile for a decode-trajectory step: ``b_p + (b_hi - b_p) * f_p**gamma`` where
+    ``f_p`` is the committed fraction of the positions before p.  A position becomes as
+    confident as the canvas ends once (nearly) all the context to its left has been
+    committed, so the canvas resolves left to right (the progression of App. A.7); a larger
+    ``gamma`` resolves fewer positions per step."""
     N = mask.numel()
     committed = (mask == 0).to(torch.float64)
     before = torch.cumsum(committed, 0) - committed
     denom = torch.arange(N, dtype=torch.float64).clamp_min(1)
-    f = torch.where(torch.arange(N) > 0, before / denom, torch.zeros(N, dtype=torch.float64))
-    return (base_b.to(torch.float64) * (1.0 + boost * f)).to(torch.float32)
+    f = torch.where(torch.arange(N) > 0, before / denom, torch.ones(N, dtype=torch.float64))
+    b = base_b.to(torch.float64)
+    return (b + (b_hi - b).clamp_min(0) * f.pow(gamma)).to(torch.float32)
 
 
 def trajectory_hidden(W: torch.Tensor, K: int, N: int, seed: int, step: int, mask: torch.Tensor,
-                      kappa: float = DEFAULT_KAPPA, targets: torch.Tensor | None = None) -> Canvas:
+                      kappa: float = DEFAULT_KAPPA, targets: torch.Tensor | None = None,
+                      gamma: float = 8.0) -> Canvas:
     """Hidden states for step ``step`` of a decode trajectory at the current ``mask``."""
     d = W.shape[1]
-    b = trajectory_profile(u_profile(N, 0.3, 4.0), mask)
+    b = trajectory_profile(u_profile(N, 0.3, 4.0), mask, gamma=gamma)
     return make_hidden(W, K, N, seed * 1000 + step, b, kappa * math.sqrt(d), flip_frac=0.1,
                        targets=targets)
