@@ -43,6 +43,7 @@ tables, the Table 4 ceilings of App. A.6 and brute force over all subsets.
 """
 from __future__ import annotations
 
+import math
 from dataclasses import dataclass
 
 import numpy as np
@@ -267,6 +268,61 @@ def readout_rows(z_rows: np.ndarray):
     return P, a, pmax, gap
 
 
+def score_positions(hidden_bits, positions, g_bits, W_bits, eps: float, tau: float, rule):
+    """Steps 1-4 for the given masked positions: per-layer readout (App. A.2), y, c, H (Eq. 1),
+    K_i, r_i, S_i (Eq. 2-4) and candidacy (Eq. 5).  Returns arrays over the canvas (entries
+    outside ``positions`` keep their "not scored" values)."""
+    hidden_bits = np.asarray(hidden_bits, dtype=np.uint16)
+    K, N, d = hidden_bits.shape
+    M = np.asarray(positions, dtype=np.int64)
+    nm = len(M)
+    out = dict(
+        layer_argmax=np.full((K, N), -1, dtype=np.int64), layer_pmax=np.full((K, N), np.nan),
+        layer_gap=np.full((K, N), np.nan), p_of_y=np.full((K, N), np.nan),
+        y=np.full(N, -1, dtype=np.int64), conf=np.full(N, np.nan), H=np.zeros(N),
+        persist=np.zeros(N, dtype=np.int64), drop=np.full(N, np.nan), stab=np.full(N, np.nan),
+        cand=np.zeros(N, dtype=bool), high=np.zeros(N, dtype=bool))
+    if nm == 0:
+        return out
+    rows = hidden_bits[:, M, :].reshape(K * nm, d)     # masked positions only (App. A.6)
+    z = project_logits(rows, g_bits, W_bits, eps).reshape(K, nm, -1)
+    for qi, i in enumerate(M):
+        P, a, pmax, gap = readout_rows(z[:, qi, :])
+        out["layer_argmax"][:, i] = a
+        out["layer_pmax"][:, i] = pmax
+        out["layer_gap"][:, i] = gap
+        yi = int(a[-1])
+        out["y"][i] = yi
+        out["p_of_y"][:, i] = P[:, yi]
+        out["conf"][i] = P[-1, yi]
+        out["H"][i] = float(entropy(P[-1]))
+        out["persist"][i] = persistence(a)
+        out["drop"][i] = confidence_drop(P[:, yi], int(out["persist"][i]))
+        out["stab"][i] = stability(int(out["persist"][i]), float(out["drop"][i]), rule["k_max"],
+                                   rule["w"])
+        out["cand"][i] = is_candidate(out["conf"][i], out["stab"][i], tau, rule["theta_c"],
+                                      rule["theta_s"])
+        out["high"][i] = bool(out["conf"][i] >= tau)
+    return out
+
+
+def _result(sc, masked, A, fb, params):
+    N = masked.shape[0]
+    commit = np.zeros(N, dtype=np.uint8)
+    for i in A:
+        commit[i] = 1
+    if fb >= 0:
+        commit[fb] = 1
+    token = np.where(commit == 1, sc["y"], -1)
+    new_mask = (masked & (commit == 0)).astype(np.uint8)
+    return StepResult(commit=commit, token=token, new_mask=new_mask, masked=masked,
+                      layer_argmax=sc["layer_argmax"], layer_pmax=sc["layer_pmax"],
+                      layer_gap=sc["layer_gap"], p_of_y=sc["p_of_y"], y=sc["y"], conf=sc["conf"],
+                      H=sc["H"], persist=sc["persist"], drop=sc["drop"], stab=sc["stab"],
+                      cand=sc["cand"], high_conf=sc["high"], accepted=A, fallback_pos=fb,
+                      params=params)
+
+
 def rpd_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, budget: float,
              rule) -> StepResult:
     """One RPD commit step for one canvas.
@@ -278,60 +334,45 @@ def rpd_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, budget: 
     """
     if isinstance(rule, str):
         rule = RULES[rule]
-    hidden_bits = np.asarray(hidden_bits, dtype=np.uint16)
-    K, N, d = hidden_bits.shape
     masked = np.asarray(mask).astype(bool)
-    M = np.nonzero(masked)[0]
-    nm = len(M)
-
-    layer_argmax = np.full((K, N), -1, dtype=np.int64)
-    layer_pmax = np.full((K, N), np.nan)
-    layer_gap = np.full((K, N), np.nan)
-    p_of_y = np.full((K, N), np.nan)
-    y = np.full(N, -1, dtype=np.int64)
-    conf = np.full(N, np.nan)
-    H = np.zeros(N)
-    persist = np.zeros(N, dtype=np.int64)
-    drop = np.full(N, np.nan)
-    stab = np.full(N, np.nan)
-    cand = np.zeros(N, dtype=bool)
-    high = np.zeros(N, dtype=bool)
-
-    if nm > 0:
-        rows = hidden_bits[:, M, :].reshape(K * nm, d)     # masked positions only (App. A.6)
-        z = project_logits(rows, g_bits, W_bits, eps).reshape(K, nm, -1)
-        for qi, i in enumerate(M):
-            P, a, pmax, gap = readout_rows(z[:, qi, :])
-            layer_argmax[:, i] = a
-            layer_pmax[:, i] = pmax
-            layer_gap[:, i] = gap
-            yi = int(a[-1])
-            y[i] = yi
-            p_of_y[:, i] = P[:, yi]
-            conf[i] = P[-1, yi]
-            H[i] = float(entropy(P[-1]))
-            persist[i] = persistence(a)
-            drop[i] = confidence_drop(P[:, yi], int(persist[i]))
-            stab[i] = stability(int(persist[i]), float(drop[i]), rule["k_max"], rule["w"])
-            cand[i] = is_candidate(conf[i], stab[i], tau, rule["theta_c"], rule["theta_s"])
-            high[i] = bool(conf[i] >= tau)
-
-    A = commit_sequential(masked, cand, H, budget)
+    sc = score_positions(hidden_bits, np.nonzero(masked)[0], g_bits, W_bits, eps, tau, rule)
+    A = commit_sequential(masked, sc["cand"], sc["H"], budget)
     fb = -1
-    if not A and nm > 0:
-        fb = fallback_commit(masked, conf, rule["window"])
-    commit = np.zeros(N, dtype=np.uint8)
-    for i in A:
-        commit[i] = 1
-    if fb >= 0:
-        commit[fb] = 1
-    token = np.where(commit == 1, y, -1)
-    new_mask = (masked & (commit == 0)).astype(np.uint8)
-    return StepResult(commit=commit, token=token, new_mask=new_mask, masked=masked,
-                      layer_argmax=layer_argmax, layer_pmax=layer_pmax, layer_gap=layer_gap,
-                      p_of_y=p_of_y, y=y, conf=conf, H=H, persist=persist, drop=drop,
-                      stab=stab, cand=cand, high_conf=high, accepted=A, fallback_pos=fb,
-                      params=dict(tau=tau, budget=budget, **rule))
+    if not A and masked.any():
+        fb = fallback_commit(masked, sc["conf"], rule["window"])
+    return _result(sc, masked, A, fb, dict(tau=tau, budget=budget, **rule))
+
+
+def active_block(masked, block: int):
+    """RPD-block (App. A.6): the active block is the first fixed block of ``block`` positions
+    that still holds a masked position; returns its masked positions (empty if none)."""
+    masked = np.asarray(masked).astype(bool)
+    idx = np.nonzero(masked)[0]
+    if len(idx) == 0:
+        return idx
+    j = int(idx[0]) // block
+    return idx[(idx >= j * block) & (idx < (j + 1) * block)]
+
+
+def rpd_block_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, rule,
+                   block: int = 32) -> StepResult:
+    """RPD-block (§3.2 "Variants", App. A.6): the candidate selection of Eq. 5 applied within
+    the active block of ``block`` positions, no cumulative-entropy budget (every candidate of
+    the block is committed), and, when no candidate passes, the most confident masked
+    position of the active block (leftmost on ties)."""
+    if isinstance(rule, str):
+        rule = RULES[rule]
+    masked = np.asarray(mask).astype(bool)
+    act = active_block(masked, block)
+    sc = score_positions(hidden_bits, act, g_bits, W_bits, eps, tau, rule)
+    A = [int(i) for i in act if sc["cand"][i]]
+    fb = -1
+    if not A and len(act):
+        fb = int(act[0])
+        for i in act[1:]:
+            if sc["conf"][i] > sc["conf"][fb]:
+                fb = int(i)
+    return _result(sc, masked, A, fb, dict(tau=tau, budget=math.inf, block=block, **rule))
 
 
 def rpd_step_batched(hidden_bits, masks, g_bits, W_bits, eps: float, taus, budgets, rule):
@@ -372,3 +413,35 @@ def step_from_scores(masked, layer_argmax, layer_p_of_y, H, tau, budget, rule):
     if fb >= 0:
         commit[fb] = 1
     return commit, cand, A, fb
+
+
+def block_step_from_scores(masked, layer_argmax, layer_p_of_y, tau, rule, block: int = 32):
+    """RPD-block's rule applied to given per-layer argmaxes and p(y_i) tables (hand-built
+    cases): returns (commit[N] uint8, cand[N] bool, fallback position)."""
+    if isinstance(rule, str):
+        rule = RULES[rule]
+    masked = np.asarray(masked).astype(bool)
+    layer_argmax = np.asarray(layer_argmax)
+    layer_p_of_y = np.asarray(layer_p_of_y, dtype=np.float64)
+    N = masked.shape[0]
+    act = active_block(masked, block)
+    cand = np.zeros(N, dtype=bool)
+    conf = np.full(N, np.nan)
+    for i in act:
+        k_i = persistence(layer_argmax[:, i])
+        r_i = confidence_drop(layer_p_of_y[:, i], k_i)
+        conf[i] = layer_p_of_y[-1, i]
+        cand[i] = is_candidate(conf[i], stability(k_i, r_i, rule["k_max"], rule["w"]), tau,
+                               rule["theta_c"], rule["theta_s"])
+    commit = np.zeros(N, dtype=np.uint8)
+    A = [int(i) for i in act if cand[i]]
+    fb = -1
+    if not A and len(act):
+        fb = int(act[0])
+        for i in act[1:]:
+            if conf[i] > conf[fb]:
+                fb = int(i)
+    commit[A] = 1
+    if fb >= 0:
+        commit[fb] = 1
+    return commit, cand, fb

@@ -184,3 +184,59 @@ def compare_step(ref: O.StepResult, got: dict, check_scores: bool = True) -> Par
     if not free:
         assert st["n_candidates"] == int(ref.cand.sum())
     return rep
+
+
+def replay_commit_rule(got: dict, masked, tau: float, budget: float, rule: dict, K: int):
+    """Apply the oracle's rule steps (Eq. 5, the sequential E_i <= beta rule and the fallback)
+    to the GPU's own per-position scores, in fp64, and return (expected commit vector, the
+    positions whose decision is within DELTA of a threshold).  This checks the scan, the
+    acceptance and the fallback at any size, independently of the projection."""
+    masked = np.asarray(masked).astype(bool)
+    N = masked.shape[0]
+    c = got["conf"].astype(np.float64)
+    S = got["stability"].astype(np.float64)
+    H = got["entropy"].astype(np.float64)
+    cand = np.zeros(N, dtype=bool)
+    near = []
+    for i in np.nonzero(masked)[0]:
+        cand[i] = O.is_candidate(c[i], S[i], tau, rule["theta_c"], rule["theta_s"])
+        if (abs(c[i] - tau) < DELTA or abs(c[i] - rule["theta_c"]) < DELTA or
+                (rule["theta_c"] <= c[i] < tau and abs(S[i] - rule["theta_s"]) < DELTA)):
+            near.append(int(i))
+    A = O.commit_sequential(masked, cand, H, budget)
+    fb = -1
+    if not A and masked.any():
+        fb = O.fallback_commit(masked, c, rule["window"])
+    commit = np.zeros(N, dtype=np.uint8)
+    commit[A] = 1
+    if fb >= 0:
+        commit[fb] = 1
+    # budget comparisons within DELTA
+    q = 0.0
+    for i in range(N):
+        if cand[i] and abs(q - budget) < DELTA:
+            near.append(int(i))
+        if masked[i] and not cand[i]:
+            q += H[i]
+    return commit, cand, near
+
+
+def compare_rows(ref_rows: dict, got: dict, positions, K: int):
+    """Per-position scores of sampled positions against the oracle's readout of their K rows.
+    ``ref_rows[i]`` = (argmax[K], pmax[K], gap[K], p_of_y[K], H_final)."""
+    worst = 0.0
+    for i in positions:
+        a, pm, gap, pyk, Hf = ref_rows[i]
+        near = np.min(gap) < DELTA
+        for k in range(K):
+            if gap[k] >= DELTA:
+                assert got["layer_argmax"][k, i] == a[k], (i, k, got["layer_argmax"][k, i], a[k])
+                worst = max(worst, abs(got["layer_pmax"][k, i] - pm[k]))
+        assert abs(got["conf"][i] - pyk[-1]) < PROB_TOL
+        assert abs(got["entropy"][i] - Hf) < PROB_TOL
+        if not near:
+            k_i = O.persistence(a)
+            assert got["persist"][i] == k_i
+            assert abs(got["drop"][i] - O.confidence_drop(pyk, k_i)) < 2 * PROB_TOL
+    assert worst < PROB_TOL
+    return worst

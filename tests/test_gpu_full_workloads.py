@@ -1,0 +1,107 @@
+"""Full-size workloads that the fp64 oracle cannot evaluate row for row in seconds.
+
+* Batched serving: 8 canvases x 1024 positions, K = 6, LLaDA-8B head, 30-100% masked
+  (~32k projected rows).  Sampled positions of every canvas are projected by the oracle and
+  compared score by score; the commitment of every canvas is checked by replaying the
+  oracle's rule on the GPU's own scores (a property that holds at any size).
+* Decode trajectory at the LLaDA-8B head shape: every step's invariants, and the full oracle
+  at the first, a middle and the last step.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import workloads as WL
+from oracle import rpd_oracle as O
+from tests.gpu_util import GpuRunner, bits
+from tests.parity import DELTA, compare_rows, compare_step, replay_commit_rule
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # collected on CPU machines, never run there
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+
+def oracle_rows(hidden_k_pos, g, W, eps):
+    """Oracle readout of one position's K rows: argmax, pmax, gap, p(y) per layer and H."""
+    z = O.project_logits(bits(hidden_k_pos), bits(g), bits(W), eps)
+    P, a, pm, gap = O.readout_rows(z)
+    y = int(a[-1])
+    return a, pm, gap, P[:, y], float(O.entropy(P[-1]))
+
+
+def test_batched_serving_full():
+    case = WL.batched_serving(seed=5)
+    K, B, N = case["K"], case["B"], case["N"]
+    runner = GpuRunner(case["W"], case["g"], K, case["eps"], rule="llada")
+    try:
+        outs = runner.step_batched(case["hidden"], case["mask"], case["tau"], case["budget"])
+    finally:
+        runner.close()
+    rule = O.RULES["llada"]
+    gen = np.random.default_rng(55)
+    for b in range(B):
+        got = outs[b]
+        masked = case["mask"][b].numpy().astype(bool)
+        st = got["stats"]
+        assert st["status"] == 0 and st["n_masked"] == int(masked.sum())
+        # commitment replayed on the GPU's own scores
+        exp, cand, near = replay_commit_rule(got, masked, case["tau"][b], case["budget"][b], rule, K)
+        gcand = got["candidate"].astype(bool)
+        for i in np.nonzero(masked)[0]:
+            if i not in near:
+                assert gcand[i] == cand[i], (b, i)
+        diff = np.nonzero(exp != got["commit"])[0]
+        if near:
+            # a decision within DELTA of its threshold may flip; everything before it may not
+            assert np.all(diff >= min(near)), (b, diff[:10], sorted(near)[:5])
+        else:
+            assert len(diff) == 0, (b, diff[:10])
+        assert np.array_equal(got["new_mask"], (masked & (got["commit"] == 0)).astype(np.uint8))
+        assert st["n_committed"] == int(got["commit"].sum()) >= 1
+        # sampled positions against the oracle
+        idx = np.nonzero(masked)[0]
+        sample = gen.choice(idx, size=min(3, len(idx)), replace=False)
+        ref_rows = {int(i): oracle_rows(case["hidden"][:, b, int(i)], case["g"], case["W"], case["eps"])
+                    for i in sample}
+        compare_rows(ref_rows, got, [int(i) for i in sample], K)
+
+
+@pytest.fixture(scope="module")
+def traj_head():
+    return WL.make_head(WL.LLADA_V, WL.LLADA_D, seed=4)
+
+
+def test_llada_trajectory(traj_head):
+    W, g = traj_head
+    K, N, V = 4, 256, WL.LLADA_V
+    gen = torch.Generator().manual_seed(4004)
+    targets = torch.randint(0, V, (N,), generator=gen)
+    runner = GpuRunner(W, g, K, 1e-6, rule="llada")
+    mask = torch.ones(N, dtype=torch.uint8)
+    checked = []
+    steps = []
+    try:
+        for t in range(64):
+            cv = WL.trajectory_hidden(W, K, N, seed=4, step=t, mask=mask, targets=targets)
+            got = runner.step(cv.hidden, mask, 0.9, 1.0)
+            m = mask.numpy().astype(bool)
+            st = got["stats"]
+            assert st["status"] == 0 and st["n_masked"] == int(m.sum())
+            assert st["n_committed"] >= 1 and np.all(got["commit"][~m] == 0)
+            assert np.array_equal(got["new_mask"], (m & (got["commit"] == 0)).astype(np.uint8))
+            steps.append((cv, mask.clone(), got))
+            mask = torch.from_numpy(got["new_mask"].copy())
+            if int(mask.sum()) <= 0.02 * N:
+                break
+    finally:
+        runner.close()
+    assert int(mask.sum()) <= 0.02 * N, "trajectory did not finish within 64 steps"
+    for t in sorted({0, len(steps) // 2, len(steps) - 1}):
+        cv, m, got = steps[t]
+        ref = O.rpd_step(bits(cv.hidden), m.numpy(), bits(g), bits(W), 1e-6, 0.9, 1.0, "llada")
+        compare_step(ref, got)
+        checked.append(t)
+    print("trajectory steps", len(steps), "oracle-checked", checked)
