@@ -38,8 +38,7 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "f33dc638adb8f691"): 1.0484e9,   # profiles/k_head_stats_llada_first_step.md
-    ("llada_tail_5_masked", "f33dc638adb8f691"): 1.0441e9,  # profiles/k_head_stats_llada_tail5.md
+    ("llada_first_step", "d3d9eb61ca56ba61"): 1.0863e9,   # profiles/k_head_stats_pair_llada_first_step.md
 }
 
 
@@ -389,7 +388,7 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
         "kernel_timing": "second timed pass of the same steps with CUDA events around each launch",
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 5 * args.steps,
+        "gpu_launches": 6 * args.steps,  # compact, gather/norm, two head tilings (one returns at once), merge, score/commit
         "clocks": clocks,
         "last_step_stats": st,
     }

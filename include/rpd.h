@@ -42,7 +42,8 @@ extern "C" {
 typedef struct rpd_ctx rpd_ctx; /* opaque, owned by the library */
 
 /* Rule parameters other than theta_h (= tau) and beta (= budget); Table 4 (App. A.6).
- * rpd_create installs the LLaDA profile: theta_c 0.6, theta_s 3.5, w 15, k_max 6, window 32.
+ * rpd_create installs the LLaDA profile: theta_c 0.6, theta_s 3.5, w 15, k_max 6, window 32,
+ * block 0.
  * The Dream profile is theta_s 2.5, w 20 with the rest unchanged. */
 typedef struct rpd_rule {
     float theta_c;  /* minimum confidence for admission through stability (Eq. 5) */
@@ -50,6 +51,13 @@ typedef struct rpd_rule {
     float w;        /* weight of the confidence-drop penalty (Eq. 4), >= 0 */
     int32_t k_max;  /* cap on prediction persistence (Eq. 4), >= 1 */
     int32_t window; /* fallback window W: first W masked positions (§3.2), >= 1 */
+    int32_t block;  /* 0: full RPD (§3.2).  > 0: RPD-block (§3.2 "Variants", App. A.6):
+                       only the active block - the first run of `block` positions (32 in
+                       the paper) that still holds a masked position - is projected and
+                       scored; every candidate in it is committed (no entropy budget;
+                       `budget` is ignored) and, if there is none, its most confident
+                       masked position.  Debug outputs outside the active block read as
+                       unmasked; rpd_stats.n_masked still counts the whole canvas. */
 } rpd_rule;
 
 /* Per-canvas step summary, written to DEVICE memory by rpd_step / rpd_step_batched. */
@@ -92,7 +100,7 @@ rpd_ctx *rpd_create(int d, int V, int K, float eps);
 int rpd_set_head(rpd_ctx *ctx, const void *W_head, const void *g_norm);
 
 /* Replace the rule parameters (Table 4).  Requires 0 <= theta_c, w >= 0, k_max >= 1,
- * window >= 1.  theta_c < tau is checked per step (Eq. 5 requires theta_c < theta_h). */
+ * window >= 1, block >= 0.  theta_c < tau is checked per step (Eq. 5 requires theta_c < theta_h). */
 int rpd_set_rule(rpd_ctx *ctx, const rpd_rule *rule);
 int rpd_get_rule(const rpd_ctx *ctx, rpd_rule *rule);
 

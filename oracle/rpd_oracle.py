@@ -340,7 +340,9 @@ def rpd_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, budget: 
     fb = -1
     if not A and masked.any():
         fb = fallback_commit(masked, sc["conf"], rule["window"])
-    return _result(sc, masked, A, fb, dict(tau=tau, budget=budget, **rule))
+    params = dict(rule)
+    params.update(tau=tau, budget=budget)
+    return _result(sc, masked, A, fb, params)
 
 
 def active_block(masked, block: int):
@@ -372,7 +374,9 @@ def rpd_block_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, ru
         for i in act[1:]:
             if sc["conf"][i] > sc["conf"][fb]:
                 fb = int(i)
-    return _result(sc, masked, A, fb, dict(tau=tau, budget=math.inf, block=block, **rule))
+    params = dict(rule)
+    params.update(tau=tau, budget=math.inf, block=block)
+    return _result(sc, masked, A, fb, params)
 
 
 def rpd_step_batched(hidden_bits, masks, g_bits, W_bits, eps: float, taus, budgets, rule):

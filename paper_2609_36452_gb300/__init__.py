@@ -30,10 +30,13 @@ RPD_ERR_UNSUPPORTED = 6
 RPD_NUM_KERNELS = 4
 KERNEL_NAMES = ("gather_norm", "head_stats", "merge", "score_commit")
 
-# Table 4 (App. A.6) rule profiles: theta_c, theta_s, w, k_max, window.
+# Table 4 (App. A.6) rule profiles: theta_c, theta_s, w, k_max, window, block (0 = full RPD;
+# 32 = the paper's RPD-block variant).
 RULE_PROFILES = {
-    "llada": (0.6, 3.5, 15.0, 6, 32),
-    "dream": (0.6, 2.5, 20.0, 6, 32),
+    "llada": (0.6, 3.5, 15.0, 6, 32, 0),
+    "dream": (0.6, 2.5, 20.0, 6, 32, 0),
+    "llada_block": (0.6, 3.5, 15.0, 6, 32, 32),
+    "dream_block": (0.6, 2.5, 20.0, 6, 32, 32),
 }
 
 lib_path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librpd.so")
@@ -41,7 +44,7 @@ lib_path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librpd.so")
 
 class RpdRule(ctypes.Structure):
     _fields_ = [("theta_c", ctypes.c_float), ("theta_s", ctypes.c_float), ("w", ctypes.c_float),
-                ("k_max", ctypes.c_int32), ("window", ctypes.c_int32)]
+                ("k_max", ctypes.c_int32), ("window", ctypes.c_int32), ("block", ctypes.c_int32)]
 
 
 class RpdStats(ctypes.Structure):
@@ -156,8 +159,9 @@ class Rpd:
         self._keep = [W, g]
         _check(rpd_set_head(self.handle, _ptr(W), _ptr(g)))
 
-    def set_rule(self, theta_c, theta_s, w, k_max, window):
-        _check(rpd_set_rule(self.handle, ctypes.byref(RpdRule(theta_c, theta_s, w, k_max, window))))
+    def set_rule(self, theta_c, theta_s, w, k_max, window, block=0):
+        _check(rpd_set_rule(self.handle,
+                            ctypes.byref(RpdRule(theta_c, theta_s, w, k_max, window, block))))
 
     def set_profile(self, name: str):
         self.set_rule(*RULE_PROFILES[name])
@@ -165,7 +169,8 @@ class Rpd:
     def get_rule(self) -> dict:
         r = RpdRule()
         _check(rpd_get_rule(self.handle, ctypes.byref(r)))
-        return dict(theta_c=r.theta_c, theta_s=r.theta_s, w=r.w, k_max=r.k_max, window=r.window)
+        return dict(theta_c=r.theta_c, theta_s=r.theta_s, w=r.w, k_max=r.k_max, window=r.window,
+                    block=r.block)
 
     def set_stream(self, stream):
         """``stream``: a torch.cuda.Stream, a raw cudaStream_t int, or None (legacy)."""

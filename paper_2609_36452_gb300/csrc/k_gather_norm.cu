@@ -31,9 +31,20 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
     __shared__ int warp_sum[32];
     __shared__ unsigned long long best_split;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    __shared__ int block_lo[kMaxBatch];  // RPD-block: first position of each canvas's active block
     pdl_wait();
     pdl_trigger();
     const int total = p.B * p.N;
+    if (p.block > 0) {
+        for (int b = tid; b < p.B; b += kCompactThreads) block_lo[b] = p.N;
+        __syncthreads();
+        for (int i = tid; i < total; i += kCompactThreads)
+            if (p.mask[i]) atomicMin(&block_lo[i / p.N], i % p.N);
+        __syncthreads();
+        for (int b = tid; b < p.B; b += kCompactThreads)
+            block_lo[b] = block_lo[b] < p.N ? (block_lo[b] / p.block) * p.block : p.N;
+        __syncthreads();
+    }
     int carry = 0;
     for (int base = 0; base < total; base += kCompactThreads * kCompactItems) {
         const int i0 = base + tid * kCompactItems;
@@ -43,6 +54,10 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
         for (int j = 0; j < kCompactItems; ++j) {
             const int i = i0 + j;
             f[j] = (i < total) ? (p.mask[i] != 0) : 0;
+            if (f[j] && p.block > 0) {
+                const int lo = block_lo[i / p.N], pos = i % p.N;
+                f[j] = pos >= lo && pos < lo + p.block;
+            }
             cnt += f[j];
         }
         const int incl = warp_inclusive_scan(cnt, lane);

@@ -125,8 +125,8 @@ __device__ __forceinline__ ScanPair block_scan_pair(ScanPair v, ScanPair *sh, Sc
     return ScanPair{base.q + incl.q - v.q, base.m + incl.m - v.m};
 }
 
-// Block-wide sums of three counters.
-__device__ __forceinline__ int3 block_sum3(int3 v, int3 *sh) {
+// Block-wide sums of four counters.
+__device__ __forceinline__ int4 block_sum4(int4 v, int4 *sh) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nwarps = (blockDim.x + 31) >> 5;
 #pragma unroll
@@ -134,14 +134,16 @@ __device__ __forceinline__ int3 block_sum3(int3 v, int3 *sh) {
         v.x += __shfl_xor_sync(0xffffffffu, v.x, o);
         v.y += __shfl_xor_sync(0xffffffffu, v.y, o);
         v.z += __shfl_xor_sync(0xffffffffu, v.z, o);
+        v.w += __shfl_xor_sync(0xffffffffu, v.w, o);
     }
     if (lane == 0) sh[warp] = v;
     __syncthreads();
-    int3 t = make_int3(0, 0, 0);
+    int4 t = make_int4(0, 0, 0, 0);
     for (int w = 0; w < nwarps; ++w) {
         t.x += sh[w].x;
         t.y += sh[w].y;
         t.z += sh[w].z;
+        t.w += sh[w].w;
     }
     return t;
 }
@@ -151,7 +153,7 @@ constexpr int kLayerBatch = 8;  // window layers whose statistics are loaded tog
 __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p) {
     constexpr int kMaxItems = kMaxCanvas / kScoreThreads;
     __shared__ ScanPair sh_scan[33];
-    __shared__ int3 sh_sum[32];
+    __shared__ int4 sh_sum[32];
     __shared__ int first_reject;
     __shared__ unsigned long long best_fb;
 
@@ -171,8 +173,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     int y[kMaxItems];
     float conf[kMaxItems], H[kMaxItems];
 
-    ScanPair local{0.f, 0};
-    int n_cand = 0;
+    ScanPair local{0.f, 0};  // (entropy of scored non-candidates, scored positions)
+    int n_cand = 0, n_masked_all = 0;
 #pragma unroll
     for (int j = 0; j < kMaxItems; ++j) {
         masked[j] = cand[j] = high[j] = false;
@@ -181,11 +183,15 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
         const int i = i0 + j;
         if (j >= items || i >= N) continue;
         const size_t pos = static_cast<size_t>(b) * N + i;
-        masked[j] = mask[i] != 0;
+        const bool is_masked = mask[i] != 0;
+        n_masked_all += is_masked;
+        // Scored positions: every masked one, or (RPD-block) the active block's masked ones,
+        // which are exactly those the compaction kept.
+        const int q = is_masked ? p.q_of_pos[pos] : -1;
+        masked[j] = q >= 0;
         int ki = 0;
         float r = 0.f, s = 0.f;
         if (masked[j]) {
-            const int q = p.q_of_pos[pos];
             // Backward over the window, a batch of layers at a time (loads issued together).
             float peak = 0.f;
             bool run = true;
@@ -259,6 +265,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     float q = pre.q;
 #pragma unroll
     for (int j = 0; j < kMaxItems; ++j) {
+        if (p.block > 0) break;  // RPD-block: no entropy budget
         if (j >= items || i0 + j >= N) break;
         if (cand[j] && q > beta) {
             atomicMin(&first_reject, i0 + j);
@@ -269,25 +276,27 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     __syncthreads();
     const int reject_at = first_reject;
 
-    int3 cnt = make_int3(0, 0, n_cand);  // accepted, accepted through c >= tau, candidates
+    // accepted, accepted through c >= tau, candidates, masked positions of the canvas
+    int4 cnt = make_int4(0, 0, n_cand, n_masked_all);
 #pragma unroll
     for (int j = 0; j < kMaxItems; ++j) {
         const bool acc = cand[j] && (i0 + j) < reject_at;
         cnt.x += acc;
         cnt.y += acc && high[j];
     }
-    const int3 tot = block_sum3(cnt, sh_sum);
-    const int total_masked = total.m;
+    const int4 tot = block_sum4(cnt, sh_sum);
+    const int total_masked = tot.w;
+    const int fallback_window = p.block > 0 ? p.block : p.window;
 
     // ------------------------------------------------------------------------ fallback
     int fb_pos = -1;
-    if (tot.x == 0 && total_masked > 0) {  // uniform across the block
+    if (tot.x == 0 && total.m > 0) {  // uniform across the block
         int rank = pre.m;
         unsigned long long mine = 0ull;
 #pragma unroll
         for (int j = 0; j < kMaxItems; ++j) {
             if (!masked[j]) continue;
-            if (rank < p.window) {
+            if (rank < fallback_window) {
                 // c >= 0: its bit pattern orders like the value; ties -> lowest position
                 const unsigned long long key =
                     (static_cast<unsigned long long>(__float_as_uint(conf[j])) << 32) |

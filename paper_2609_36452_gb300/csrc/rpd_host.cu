@@ -83,7 +83,7 @@ struct rpd_ctx {
     float eps = 0.f;
     int device = 0, num_sms = 0;
     const void *W = nullptr, *g = nullptr;
-    rpd_rule rule{0.6f, 3.5f, 15.0f, 6, 32};
+    rpd_rule rule{0.6f, 3.5f, 15.0f, 6, 32, 0};
     cudaStream_t stream = nullptr;
     rpd_debug dbg{};
 
@@ -210,6 +210,7 @@ int check_rule(const rpd_rule &r) {
         return fail(RPD_ERR_INVALID_ARGUMENT, "w must be finite and >= 0");
     if (r.k_max < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "k_max must be >= 1");
     if (r.window < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "window must be >= 1");
+    if (r.block < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "block must be >= 0");
     return RPD_OK;
 }
 
@@ -250,7 +251,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         KernelTimer t(c, 0);
         CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
                          num_n, c->max_splits, c->num_sms, pair_slots,
-                         head_stream_in_tiles(c->V, c->d, c->num_sms)};
+                         head_stream_in_tiles(c->V, c->d, c->num_sms), c->rule.block};
         e = launch_compact(cp, c->stream);
         if (e == cudaSuccess) {
             NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
@@ -298,6 +299,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         sp.w = c->rule.w;
         sp.k_max = c->rule.k_max;
         sp.window = c->rule.window;
+        sp.block = c->rule.block;
         for (int b = 0; b < B; ++b) {
             sp.tau[b] = tau[b];
             sp.budget[b] = budget[b];

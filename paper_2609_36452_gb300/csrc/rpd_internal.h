@@ -55,6 +55,7 @@ struct CompactParams {
     int single_slots;     // CTAs of the single-CTA head kernel
     int pair_slots;       // CTA pairs of the pair head kernel (0: pair tiles unavailable)
     float hbm_tiles;      // time to stream the head once, in single-CTA tile times
+    int block;            // 0: every masked position; > 0: only each canvas's active block
 };
 
 // Relative cost of a CTA-pair tile (256 rows on two SMs) against a single-CTA tile (128 rows
@@ -115,6 +116,7 @@ struct ScoreParams {
     int B, N, K;
     float theta_c, theta_s, w;
     int k_max, window;
+    int block;                  // 0: full RPD; > 0: RPD-block (no budget, in-block fallback)
     float tau[kMaxBatch];
     float budget[kMaxBatch];
 };

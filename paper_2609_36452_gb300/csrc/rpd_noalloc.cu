@@ -140,7 +140,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
                                 uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats,
                                 void *stream_ptr) {
     char msg[256];
-    const rpd_rule rule = rule_in ? *rule_in : rpd_rule{0.6f, 3.5f, 15.0f, 6, 32};
+    const rpd_rule rule = rule_in ? *rule_in : rpd_rule{0.6f, 3.5f, 15.0f, 6, 32, 0};
     if (d < 64 || d % 8 != 0) return na_fail(RPD_ERR_INVALID_ARGUMENT, "d must be a multiple of 8 and >= 64");
     if (d > kNaMaxD) {
         snprintf(msg, sizeof(msg), "rpd_step_noalloc: d=%d exceeds the static arena limit %d", d, kNaMaxD);
@@ -157,7 +157,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     }
     if (!(eps >= 0.f) || !std::isfinite(eps)) return na_fail(RPD_ERR_INVALID_ARGUMENT, "eps must be finite and >= 0");
     if (!(rule.theta_c >= 0.f) || !(rule.w >= 0.f) || rule.k_max < 1 || rule.window < 1 ||
-        std::isnan(rule.theta_s))
+        rule.block < 0 || std::isnan(rule.theta_s))
         return na_fail(RPD_ERR_INVALID_ARGUMENT, "invalid rule");
     if (!(tau > 0.f && tau <= 1.f) || !(rule.theta_c < tau))
         return na_fail(RPD_ERR_INVALID_ARGUMENT, "tau must be in (0, 1] and above theta_c");
@@ -201,7 +201,8 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     cudaError_t e = cudaMemsetAsync(meta, 0, kMetaWords * 4, stream);
     if (e == cudaSuccess) {
         CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n, splits,
-                         dev->num_sms, pair_slots, head_stream_in_tiles(V, d, dev->num_sms)};
+                         dev->num_sms, pair_slots, head_stream_in_tiles(V, d, dev->num_sms),
+                         rule.block};
         e = launch_compact(cp, stream);
     }
     if (e == cudaSuccess) {
@@ -240,6 +241,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         sp.w = rule.w;
         sp.k_max = rule.k_max;
         sp.window = rule.window;
+        sp.block = rule.block;
         sp.tau[0] = tau;
         sp.budget[0] = budget;
         e = launch_score_commit(sp, stream);

@@ -30,7 +30,8 @@ class GpuRunner:
         if isinstance(rule, str):
             self.ctx.set_profile(rule)
         else:
-            self.ctx.set_rule(rule["theta_c"], rule["theta_s"], rule["w"], rule["k_max"], rule["window"])
+            self.ctx.set_rule(rule["theta_c"], rule["theta_s"], rule["w"], rule["k_max"], rule["window"],
+                              rule.get("block", 0))
 
     def _alloc(self, B, N):
         dev, K = self.dev, self.K

@@ -240,3 +240,61 @@ def compare_rows(ref_rows: dict, got: dict, positions, K: int):
             assert abs(got["drop"][i] - O.confidence_drop(pyk, k_i)) < 2 * PROB_TOL
     assert worst < PROB_TOL
     return worst
+
+
+def compare_block_step(ref: O.StepResult, got: dict) -> ParityReport:
+    """RPD-block: scores of the active block's positions, and the commit set against every
+    outcome the oracle admits under its near-threshold decisions (same tolerances as
+    compare_step; no budget is involved)."""
+    rep = ParityReport()
+    scored = np.isfinite(ref.conf)
+    idx = np.nonzero(scored)[0]
+    rep.n_masked = int(ref.masked.sum())
+    K = ref.layer_argmax.shape[0]
+    p = ref.params
+    free = [i for i in near_threshold_positions(ref) if scored[i]]
+    rep.near_threshold = free
+    if len(idx):
+        rep.max_dconf = float(np.max(np.abs(got["conf"][idx] - ref.conf[idx])))
+        rep.max_dH = float(np.max(np.abs(got["entropy"][idx] - ref.H[idx])))
+        assert rep.max_dconf < PROB_TOL and rep.max_dH < PROB_TOL
+        for i in idx:
+            for k in range(K):
+                if ref.layer_gap[k, i] >= DELTA:
+                    assert got["layer_argmax"][k, i] == ref.layer_argmax[k, i], (k, i)
+            if i not in free:
+                assert bool(got["candidate"][i]) == bool(ref.cand[i]), i
+    # positions outside the active block are not scored and never committed
+    outside = ref.masked & ~scored
+    assert np.all(got["candidate"][outside] == 0) and np.all(got["commit"][outside] == 0)
+    if len(free) > MAX_FREE:
+        raise AssertionError("too many near-threshold decisions: parity unpinned for this case")
+    adm = set()
+    for flips in itertools.product([False, True], repeat=len(free)):
+        cand = ref.cand.copy()
+        for f, pos in zip(flips, free):
+            if f:
+                cand[pos] = not cand[pos]
+        A = tuple(int(i) for i in idx if cand[i])
+        if A:
+            adm.add(A)
+        elif len(idx):
+            cbest = max(ref.conf[i] for i in idx)
+            for i in idx:
+                if ref.conf[i] >= cbest * (1 - FALLBACK_REL):
+                    adm.add((int(i),))
+        else:
+            adm.add(())
+    rep.admissible = len(adm)
+    commit = np.asarray(got["commit"]).astype(np.uint8)
+    cset = tuple(int(i) for i in np.nonzero(commit)[0])
+    assert cset in adm, (cset, sorted(adm)[:5])
+    for i in cset:
+        if ref.layer_gap[K - 1, i] >= DELTA:
+            assert got["token"][i] == ref.y[i]
+    assert np.array_equal(got["new_mask"], (ref.masked & (commit == 0)).astype(np.uint8))
+    st = got["stats"]
+    assert st["status"] == 0 and st["n_masked"] == rep.n_masked
+    assert st["n_committed"] == len(cset)
+    assert st["n_high_conf"] + st["n_stability"] + st["fallback_used"] == st["n_committed"]
+    return rep

@@ -24,12 +24,17 @@ if not torch.cuda.is_available():  # collected on CPU machines, never run there
     pytest.skip("needs a CUDA GPU", allow_module_level=True)
 
 
-def oracle_rows(hidden_k_pos, g, W, eps):
-    """Oracle readout of one position's K rows: argmax, pmax, gap, p(y) per layer and H."""
-    z = O.project_logits(bits(hidden_k_pos), bits(g), bits(W), eps)
-    P, a, pm, gap = O.readout_rows(z)
-    y = int(a[-1])
-    return a, pm, gap, P[:, y], float(O.entropy(P[-1]))
+def oracle_rows(hidden_rows, g, W, eps):
+    """Oracle readout of several positions' K rows (``hidden_rows`` [P][K][d]): per position
+    argmax, pmax, gap, p(y) per layer and the final entropy; one projection for all rows."""
+    P_, K, d = hidden_rows.shape
+    z = O.project_logits(bits(hidden_rows.reshape(P_ * K, d)), bits(g), bits(W), eps)
+    out = []
+    for j in range(P_):
+        P, a, pm, gap = O.readout_rows(z[j * K:(j + 1) * K])
+        y = int(a[-1])
+        out.append((a, pm, gap, P[:, y], float(O.entropy(P[-1]))))
+    return out
 
 
 def test_batched_serving_full():
@@ -42,6 +47,13 @@ def test_batched_serving_full():
         runner.close()
     rule = O.RULES["llada"]
     gen = np.random.default_rng(55)
+    samples = {}
+    for b in range(B):
+        idx = np.nonzero(case["mask"][b].numpy())[0]
+        samples[b] = [int(i) for i in gen.choice(idx, size=min(3, len(idx)), replace=False)]
+    picks = [(b, i) for b in range(B) for i in samples[b]]
+    rows = torch.stack([case["hidden"][:, b, i] for b, i in picks])    # [P][K][d]
+    readouts = dict(zip(picks, oracle_rows(rows, case["g"], case["W"], case["eps"])))
     for b in range(B):
         got = outs[b]
         masked = case["mask"][b].numpy().astype(bool)
@@ -62,11 +74,8 @@ def test_batched_serving_full():
         assert np.array_equal(got["new_mask"], (masked & (got["commit"] == 0)).astype(np.uint8))
         assert st["n_committed"] == int(got["commit"].sum()) >= 1
         # sampled positions against the oracle
-        idx = np.nonzero(masked)[0]
-        sample = gen.choice(idx, size=min(3, len(idx)), replace=False)
-        ref_rows = {int(i): oracle_rows(case["hidden"][:, b, int(i)], case["g"], case["W"], case["eps"])
-                    for i in sample}
-        compare_rows(ref_rows, got, [int(i) for i in sample], K)
+        ref_rows = {i: readouts[(b, i)] for i in samples[b]}
+        compare_rows(ref_rows, got, samples[b], K)
 
 
 @pytest.fixture(scope="module")

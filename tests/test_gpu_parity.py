@@ -13,7 +13,7 @@ import torch
 import workloads as WL
 from oracle import rpd_oracle as O
 from tests.gpu_util import GpuRunner, bits
-from tests.parity import compare_step
+from tests.parity import compare_block_step, compare_step
 
 pytestmark = pytest.mark.gpu
 
@@ -259,4 +259,69 @@ def test_dream_mid_decode_full():
     Dream rule profile."""
     case = WL.dream_mid_decode(seed=3)
     ref, got, rep = run_and_compare(case)
+    print(rep, got["stats"])
+
+
+# ----------------------------------------------------------------------------- RPD-block
+
+def block_rule(block, base="llada"):
+    return dict(O.RULES[base], block=block)
+
+
+@pytest.mark.parametrize("block,prefix", [(32, 0), (32, 40), (16, 70), (8, 3)])
+def test_rpd_block_matches_oracle(block, prefix):
+    """RPD-block on a calibrated canvas whose first ``prefix`` positions are committed: the
+    active block is the first one still holding a masked position."""
+    case = small_case(91 + block + prefix, K=4, N=128, a=torch.ones(4), flip=0.15)
+    mask = case["mask"].clone()
+    mask[:prefix] = 0
+    rule = block_rule(block)
+    runner = GpuRunner(case["W"], case["g"], case["K"], case["eps"], rule=rule)
+    try:
+        got = runner.step(case["hidden"], mask, case["tau"], case["budget"])
+    finally:
+        runner.close()
+    ref = O.rpd_block_step(bits(case["hidden"]), mask.numpy(), bits(case["g"]), bits(case["W"]),
+                           case["eps"], case["tau"], rule, block=block)
+    rep = compare_block_step(ref, got)
+    print(rep, got["stats"])
+
+
+def test_rpd_block_batched_canvases():
+    K, N, d, V, B = 3, 96, 256, 2048, 3
+    W, g = WL.make_head(V, d, 92, w_std=0.08)
+    hidden = torch.empty(K, B, N, d, dtype=torch.bfloat16)
+    masks = torch.ones(B, N, dtype=torch.uint8)
+    for b in range(B):
+        cv = WL.make_hidden(W, K, N, 800 + b, WL.u_profile(N, 0.5, 3.0),
+                            WL.calibrated_sigma(V, d, 0.08, 3.0), flip_frac=0.1)
+        hidden[:, b] = cv.hidden
+    masks[1, :33] = 0   # canvas 1: active block starts at 32
+    masks[2, :] = 0     # canvas 2: nothing masked
+    rule = block_rule(32)
+    runner = GpuRunner(W, g, K, rule=rule)
+    try:
+        outs = runner.step_batched(hidden, masks, [0.9] * B, [1.0] * B)
+    finally:
+        runner.close()
+    for b in range(B):
+        ref = O.rpd_block_step(bits(hidden[:, b]), masks[b].numpy(), bits(g), bits(W), 1e-6, 0.9,
+                               rule, block=32)
+        compare_block_step(ref, outs[b])
+    assert outs[2]["stats"]["n_committed"] == 0
+
+
+def test_rpd_block_llada_first_step_full(llada_head):
+    """RPD-block at the LLaDA-8B head shape: only the first 32 positions are projected."""
+    W, g = llada_head
+    case = WL.llada_first_step(seed=2, W=W, g=g)
+    rule = block_rule(32)
+    runner = GpuRunner(W, g, case["K"], case["eps"], rule=rule)
+    try:
+        got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+    finally:
+        runner.close()
+    ref = O.rpd_block_step(bits(case["hidden"]), case["mask"].numpy(), bits(g), bits(W),
+                           case["eps"], case["tau"], rule, block=32)
+    rep = compare_block_step(ref, got)
     print(rep, got["stats"])
