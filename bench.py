@@ -214,10 +214,51 @@ def run_reference(args):
 
 
 def config_dict(case, R):
-    return {"workload": case["name"], "batch": 1, "N": case["N"], "K": case["K"],
+    B = case.get("B", 1)
+    rule = case["rule"]
+    return {"workload": case["name"], "batch": B, "N": case["N"], "K": case["K"],
             "d": case["d"], "V": case["V"], "rows": R, "tau": case["tau"], "budget": case["budget"],
-            "rule": "llada (Table 4)", "signal_kappa": case.get("kappa"),
-            "l2": "inputs larger than L2: the 1.04 GB head is streamed every step"}
+            "rule": f"{rule} (Table 4)" if "block" not in rule else f"{rule} (Table 4, RPD-block 32)",
+            "signal_kappa": case.get("kappa"),
+            "l2": f"inputs larger than L2: the {2 * case['V'] * case['d'] / 1e9:.2f} GB head is streamed every step"}
+
+
+def load_workload(args, rank):
+    """The benchmarked workload for this rank (each rank draws its own canvases)."""
+    import workloads as WL
+    if args.workload == "llada_first_step":
+        case = make_workload(rank, args.masked)
+    elif args.workload == "dream_mid_decode":
+        case = WL.dream_mid_decode(seed=3 + 97 * rank)
+    elif args.workload == "batched_serving":
+        case = WL.batched_serving(seed=5 + 97 * rank)
+    else:
+        raise ValueError(args.workload)
+    if args.block:
+        case["rule"] = case["rule"] + "_block"
+        case["name"] = case["name"] + "_rpd_block"
+    return case
+
+
+def masked_rows(case):
+    """Projected rows of one step: K x masked positions (RPD-block: the active blocks only)."""
+    import workloads as WL  # noqa: F401
+    masks = case["mask"].reshape(-1, case["N"])
+    rows = 0
+    for m in masks:
+        idx = torch.nonzero(m).flatten()
+        if "block" in case["rule"] and len(idx):
+            lo = (int(idx[0]) // 32) * 32
+            idx = idx[(idx >= lo) & (idx < lo + 32)]
+        rows += case["K"] * len(idx)
+    return rows
+
+
+def aggregate_timing(ms_total_local: float, steps: int, world: int, reduce_max):
+    """Whole-job timing: the slowest rank's time for ``steps`` steps on every rank, and the
+    aggregate throughput (every rank ran its own canvases)."""
+    ms_total = float(reduce_max(ms_total_local))
+    return ms_total, ms_total / steps, world * steps / (ms_total / 1e3)
 
 
 def run_rpd(args):
@@ -229,32 +270,46 @@ def run_rpd(args):
         dist.init_process_group("nccl", device_id=dev)
     import paper_2609_36452_gb300 as rpd
 
-    case = make_workload(rank, args.masked)
+    case = load_workload(args, rank)
     K, N, d, V = case["K"], case["N"], case["d"], case["V"]
-    R, flops, bytes_ = work_per_step(case)
+    B = case.get("B", 1)
+    R = masked_rows(case)
+    flops = 2.0 * R * d * V
+    bytes_ = 2.0 * V * d + 2.0 * R * d
     W = case["W"].to(dev)
     g = case["g"].to(dev)
     hidden = case["hidden"].to(dev).contiguous()
     mask0 = case["mask"].to(dev)
     mask = mask0.clone()
-    commit = torch.zeros(N, dtype=torch.uint8, device=dev)
-    token = torch.full((N,), -1, dtype=torch.int32, device=dev)
-    stats = torch.zeros(8, dtype=torch.int32, device=dev)
+    commit = torch.zeros(B, N, dtype=torch.uint8, device=dev)
+    token = torch.full((B, N), -1, dtype=torch.int32, device=dev)
+    stats = torch.zeros(B, 8, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     ctx = rpd.Rpd(d, V, K, case["eps"])
     ctx.set_head(W, g)
     ctx.set_profile(case["rule"])
     ctx.set_stream(stream)
-    ctx.reserve(1, N)
+    ctx.reserve(B, N)
 
     def step():
         mask.copy_(mask0, non_blocking=True)
-        ctx.step(hidden, mask, case["tau"], case["budget"], commit, token, stats)
+        if B == 1:
+            ctx.step(hidden, mask.reshape(N), case["tau"], case["budget"], commit[0], token[0], stats[0])
+        else:
+            ctx.step_batched(hidden, mask, case["tau"], case["budget"], commit, token, stats)
 
     def barrier():
         if world > 1:
             import torch.distributed as dist
             dist.barrier()
+
+    def reduce_max(x):
+        if world == 1:
+            return x
+        import torch.distributed as dist
+        t = torch.tensor([x], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
 
     sampler = ClockSampler(local) if rank == 0 else None
     if sampler:
@@ -262,8 +317,8 @@ def run_rpd(args):
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize(dev)
-    st = rpd.stats_dict(stats.cpu())
-    assert st["status"] == 0, st
+    st = [rpd.stats_dict(stats[b].cpu()) for b in range(B)]
+    assert all(x["status"] == 0 for x in st), st
 
     # Timed pass 1: the step time (no per-kernel events, which would serialise the
     # programmatic-dependent-launch overlap between the step's kernels).
@@ -277,7 +332,7 @@ def run_rpd(args):
     e1.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
-    ms_total = e0.elapsed_time(e1)
+    ms_local = e0.elapsed_time(e1)
     # Timed pass 2: the same K steps with CUDA events around every launch on the context's
     # stream, for per-kernel durations (the roofline of the dominant kernel).
     ctx.kernel_times(reset=True)
@@ -288,18 +343,12 @@ def run_rpd(args):
     ctx.profile(False)
     clocks = sampler.stop() if sampler else None
     ktimes = ctx.kernel_times(reset=True)
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms_total], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
-    ms_step = ms_total / args.steps
-    steps_s = world * args.steps / (ms_total / 1e3)
+    ms_total, ms_step, steps_s = aggregate_timing(ms_local, args.steps, world, reduce_max)
 
     # ---------------------------------------------------------------- end to end (host buffers)
     e2e = None
-    if not args.no_e2e:
-        e2e = measure_e2e(ctx, case, args, world, barrier, dev)
+    if not args.no_e2e and B == 1:
+        e2e = measure_e2e(ctx, case, args, world, barrier, reduce_max)
 
     if rank != 0:
         ctx.close()
@@ -307,18 +356,19 @@ def run_rpd(args):
             import torch.distributed as dist
             dist.destroy_process_group()
         return
-    emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st, world)
+    emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e,
+         st[0] if B == 1 else st, world)
     ctx.close()
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
 
 
-def measure_e2e(ctx, case, args, world, barrier, dev):
+def measure_e2e(ctx, case, args, world, barrier, reduce_max):
     """Same step through rpd_step_host: pinned host inputs copied in, results read back."""
     N = case["N"]
-    hid_h = case["hidden"].contiguous().pin_memory()
-    mask_h0 = case["mask"].clone()
+    hid_h = case["hidden"].reshape(case["K"], N, case["d"]).contiguous().pin_memory()
+    mask_h0 = case["mask"].reshape(N).clone()
     mask_h = mask_h0.clone().pin_memory()
     commit_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
     token_h = torch.full((N,), -1, dtype=torch.int32).pin_memory()
@@ -332,12 +382,7 @@ def measure_e2e(ctx, case, args, world, barrier, dev):
     for _ in range(e2e_steps):
         mask_h.copy_(mask_h0)
         ctx.step_host(hid_h, mask_h, case["tau"], case["budget"], commit_h, token_h, stats_h)
-    e2e_s = time.perf_counter() - t0
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = reduce_max(time.perf_counter() - t0)
     h2d = hid_h.numel() * 2 + N + N * 4
     d2h = N + N + N * 4 + 32
     return {"value": e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
@@ -369,7 +414,7 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
     roof["algorithmic_flops"] = flops
 
     cpu = None
-    if not args.no_cpu_baseline and world >= 1:
+    if not args.no_cpu_baseline and case.get("B", 1) == 1 and "block" not in case["rule"]:
         r_rows, dt, threads = cpu_oracle_rate(case, args.cpu_positions)
         cpu = {"value": r_rows / R, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"oracle step over the first {args.cpu_positions} of 256 masked positions "
@@ -477,7 +522,9 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["rpd", "reference"], default="rpd")
-    ap.add_argument("--workload", choices=["llada_first_step", "trajectory"], default="llada_first_step")
+    ap.add_argument("--workload", choices=["llada_first_step", "dream_mid_decode", "batched_serving",
+                                           "trajectory"], default="llada_first_step")
+    ap.add_argument("--block", action="store_true", help="RPD-block rule (blocks of 32)")
     ap.add_argument("--cpu-positions", type=int, default=32)
     ap.add_argument("--ref-positions", type=int, default=8)
     ap.add_argument("--ref-seconds", type=float, default=150.0)
