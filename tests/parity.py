@@ -102,7 +102,7 @@ def admissible_commits(ref: O.StepResult, free_positions):
 def near_threshold_positions(ref: O.StepResult):
     p = ref.params
     out = []
-    for i in np.nonzero(ref.masked)[0]:
+    for i in np.nonzero(ref.masked & np.isfinite(ref.conf))[0]:   # scored positions
         c, s = ref.conf[i], ref.stab[i]
         near = abs(c - p["tau"]) < DELTA or abs(c - p["theta_c"]) < DELTA
         if p["theta_c"] - DELTA <= c < p["tau"] + DELTA and abs(s - p["theta_s"]) < DELTA:
