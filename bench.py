@@ -220,6 +220,8 @@ def config_dict(case, R):
             "d": case["d"], "V": case["V"], "rows": R, "tau": case["tau"], "budget": case["budget"],
             "rule": f"{rule} (Table 4)" if "block" not in rule else f"{rule} (Table 4, RPD-block 32)",
             "signal_kappa": case.get("kappa"),
+            "projection": "lazy" if "lazy_rows" in case else "all window layers",
+            "rows_projected": case.get("lazy_rows", R),
             "l2": f"inputs larger than L2: the {2 * case['V'] * case['d'] / 1e9:.2f} GB head is streamed every step"}
 
 
@@ -283,13 +285,14 @@ def run_rpd(args):
     mask = mask0.clone()
     commit = torch.zeros(B, N, dtype=torch.uint8, device=dev)
     token = torch.full((B, N), -1, dtype=torch.int32, device=dev)
-    stats = torch.zeros(B, 8, dtype=torch.int32, device=dev)
+    stats = torch.zeros(B, rpd.STATS_WORDS, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     ctx = rpd.Rpd(d, V, K, case["eps"])
     ctx.set_head(W, g)
     ctx.set_profile(case["rule"])
     ctx.set_stream(stream)
     ctx.reserve(B, N)
+    ctx.set_projection(args.projection)
 
     def step():
         mask.copy_(mask0, non_blocking=True)
@@ -319,6 +322,17 @@ def run_rpd(args):
     torch.cuda.synchronize(dev)
     st = [rpd.stats_dict(stats[b].cpu()) for b in range(B)]
     assert all(x["status"] == 0 for x in st), st
+    if args.projection != "all":
+        # Lazy projection: the work is data dependent - the rows actually projected, and one
+        # head stream per pass (two when the band is not empty).
+        nmt = sum(int(torch.count_nonzero(m)) for m in case["mask"].reshape(-1, N))
+        rows_done = st[0]["n_rows"]
+        passes = 1 if rows_done in (nmt, K * nmt) else 2
+        flops = 2.0 * rows_done * d * V
+        bytes_ = passes * 2.0 * V * d + 2.0 * rows_done * d
+        case["name"] = case["name"] + "_" + args.projection
+        case["lazy_rows"] = rows_done
+        case["lazy_passes"] = passes
 
     # Timed pass 1: the step time (no per-kernel events, which would serialise the
     # programmatic-dependent-launch overlap between the step's kernels).
@@ -372,7 +386,7 @@ def measure_e2e(ctx, case, args, world, barrier, reduce_max):
     mask_h = mask_h0.clone().pin_memory()
     commit_h = torch.zeros(N, dtype=torch.uint8).pin_memory()
     token_h = torch.full((N,), -1, dtype=torch.int32).pin_memory()
-    stats_h = torch.zeros(8, dtype=torch.int32).pin_memory()
+    stats_h = torch.zeros(9, dtype=torch.int32).pin_memory()
     e2e_steps = max(3, min(args.steps, 200))
     for _ in range(2):
         mask_h.copy_(mask_h0)
@@ -393,7 +407,8 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
     K = case["K"]
     peaks = load_peaks()
     head_ms, head_n = ktimes["head_stats"]
-    head_avg_ms = head_ms / max(head_n, 1)
+    # head-statistics time per step (a lazy step runs one head pass per projection pass)
+    head_avg_ms = head_ms / max(args.steps, 1)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
     t_hbm = bytes_ / (peaks["hbm_gbs"] * 1e9)
     if t_tc >= t_hbm:
@@ -429,8 +444,8 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
         "rows_per_s": steps_s * R,
         "roofline": roof,
         "step_roofline_frac": step_roof,
-        "kernels_ms": {k: (v[0] / max(v[1], 1)) for k, v in ktimes.items()},
-        "kernel_timing": "second timed pass of the same steps with CUDA events around each launch",
+        "kernels_ms": {k: v[0] / max(args.steps, 1) for k, v in ktimes.items()},
+        "kernel_timing": "per step; second timed pass of the same steps with CUDA events around each launch",
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": 6 * args.steps,  # compact, gather/norm, two head tilings (one returns at once), merge, score/commit
@@ -462,14 +477,15 @@ def run_trajectory(args):
     stream = torch.cuda.current_stream(dev)
     ctx.set_stream(stream)
     ctx.reserve(1, N)
+    ctx.set_projection(args.projection)
     peaks = load_peaks()
     hidden_d = torch.empty(K, N, d, dtype=torch.bfloat16, device=dev)
     mask_d = torch.empty(N, dtype=torch.uint8, device=dev)
     commit = torch.zeros(N, dtype=torch.uint8, device=dev)
     token = torch.full((N,), -1, dtype=torch.int32, device=dev)
-    stats = torch.zeros(8, dtype=torch.int32, device=dev)
+    stats = torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev)
 
-    def trajectory(record):
+    def trajectory(record):  # noqa: ARG001
         mask = torch.ones(N, dtype=torch.uint8)
         steps = []
         for t in range(64):
@@ -487,11 +503,12 @@ def run_trajectory(args):
             st = rpd.stats_dict(stats.cpu())
             assert st["status"] == 0 and st["n_masked"] == nm, st
             ms = e0.elapsed_time(e1)
-            R = K * nm
+            R = st["n_rows"]                      # rows actually projected (lazy: data dependent)
+            passes = 1 if R in (nm, K * nm) else 2  # head streams (one unless a band pass ran)
             roof_s = max(2.0 * R * d * V / (peaks["bf16_tflops"] * 1e12),
-                         (2.0 * V * d + 2.0 * R * d) / (peaks["hbm_gbs"] * 1e9))
-            steps.append({"t": t, "masked": nm, "committed": st["n_committed"], "ms": ms,
-                          "roofline_ms": roof_s * 1e3})
+                         (passes * 2.0 * V * d + 2.0 * R * d) / (peaks["hbm_gbs"] * 1e9))
+            steps.append({"t": t, "masked": nm, "committed": st["n_committed"], "rows": R,
+                          "ms": ms, "roofline_ms": roof_s * 1e3})
             mask = mask_d.cpu()
             if int(mask.sum()) <= 0.02 * N:
                 break
@@ -506,7 +523,8 @@ def run_trajectory(args):
     total_ms = sum(s["ms"] for s in steps)
     roof_ms = sum(s["roofline_ms"] for s in steps)
     out = {
-        "metric": METRIC, "workload": "llada_trajectory", "value": len(steps) / (total_ms / 1e3),
+        "metric": METRIC, "workload": "llada_trajectory" + ("" if args.projection == "all" else "_" + args.projection),
+        "value": len(steps) / (total_ms / 1e3),
         "unit": UNIT, "n_gpus": 1, "steps": len(steps), "total_ms": total_ms,
         "trajectory_roofline_frac": roof_ms / total_ms, "remaining_masked": steps[-1]["masked"] - steps[-1]["committed"],
         "kernels_ms_total": {k: v[0] for k, v in kt.items()},
@@ -525,6 +543,9 @@ def main():
     ap.add_argument("--workload", choices=["llada_first_step", "dream_mid_decode", "batched_serving",
                                            "trajectory"], default="llada_first_step")
     ap.add_argument("--block", action="store_true", help="RPD-block rule (blocks of 32)")
+    ap.add_argument("--projection", choices=["all", "lazy", "auto"], default="all",
+                    help="window layers projected: all (the step as defined), lazy (earlier "
+                         "layers only for band positions), auto (chosen per step on the device)")
     ap.add_argument("--cpu-positions", type=int, default=32)
     ap.add_argument("--ref-positions", type=int, default=8)
     ap.add_argument("--ref-seconds", type=float, default=150.0)

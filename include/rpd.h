@@ -70,6 +70,10 @@ typedef struct rpd_stats {
     int32_t fallback_used;/* 1 if A_t was empty and the fallback commit was made */
     int32_t fallback_pos; /* canvas index of the fallback commit, -1 if none */
     int32_t status;       /* RPD_OK, or RPD_ERR_TIMEOUT if a kernel's bounded wait ran out */
+    int32_t n_rows;       /* hidden-state rows projected through the head by this call (all
+                             canvases): K x scored positions, or with lazy projection the
+                             final layer of every scored position plus the earlier window
+                             layers of the band positions */
 } rpd_stats;
 
 /* Optional per-position outputs (DEVICE pointers; any may be NULL).  Layouts use the
@@ -110,6 +114,24 @@ int rpd_set_stream(rpd_ctx *ctx, void *stream);
 /* Pre-size scratch for B canvases of N positions, so that later steps of that size
  * allocate nothing.  Steps grow scratch on demand otherwise (synchronising the device). */
 int rpd_reserve(rpd_ctx *ctx, int B, int N);
+
+/* How the window layers are projected (App. A.6, "Layerwise projection").
+ *   RPD_PROJECT_ALL (default): every window layer of every scored position, in one pass over
+ *     the head.
+ *   RPD_PROJECT_LAZY: a first pass projects the final layer of every scored position; a second
+ *     pass projects the earlier window layers only of the positions whose final confidence lies
+ *     in the stability band theta_c <= c < tau - the only positions whose candidacy depends on
+ *     K_i and r_i (Eq. 5).  Commits, tokens, confidences and entropies are the same as with
+ *     RPD_PROJECT_ALL; the head is streamed twice when the band is not empty.  Debug outputs
+ *     of positions outside the band report persist 0, drop 0, stability 0 and, for layers
+ *     below the final one, layer_argmax -1 and layer_pmax 0. */
+#define RPD_PROJECT_ALL 0
+#define RPD_PROJECT_LAZY 1
+/*   RPD_PROJECT_AUTO: per step, on the device, lazy when its two passes are estimated cheaper
+ *     than one pass over every layer (many scored positions: the contraction is bound by the
+ *     tensor cores), otherwise every layer (few positions: bound by streaming the head). */
+#define RPD_PROJECT_AUTO 2
+int rpd_set_projection(rpd_ctx *ctx, int mode);
 
 /* Install (or with NULL, clear) the optional per-position outputs. */
 int rpd_set_debug(rpd_ctx *ctx, const rpd_debug *debug);

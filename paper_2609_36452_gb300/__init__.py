@@ -15,7 +15,7 @@ __all__ = [
     "RPD_OK", "RPD_ERR_INVALID_ARGUMENT", "RPD_ERR_NO_HEAD", "RPD_ERR_CUDA",
     "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
-    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_step",
+    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_profile_enable", "rpd_kernel_times",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
@@ -50,7 +50,7 @@ class RpdRule(ctypes.Structure):
 class RpdStats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "n_masked", "n_candidates", "n_high_conf", "n_stability", "n_committed",
-        "fallback_used", "fallback_pos", "status")]
+        "fallback_used", "fallback_pos", "status", "n_rows")]
 
 
 class RpdDebug(ctypes.Structure):
@@ -60,6 +60,11 @@ class RpdDebug(ctypes.Structure):
 
 
 STATS_FIELDS = [f[0] for f in RpdStats._fields_]
+STATS_WORDS = len(STATS_FIELDS)  # int32 words of one rpd_stats
+RPD_PROJECT_ALL = 0
+RPD_PROJECT_LAZY = 1
+RPD_PROJECT_AUTO = 2
+PROJECTION_MODES = {"all": RPD_PROJECT_ALL, "lazy": RPD_PROJECT_LAZY, "auto": RPD_PROJECT_AUTO}
 
 
 class RpdError(RuntimeError):
@@ -83,6 +88,7 @@ def _load():
         "rpd_set_stream": (i32, [vp, vp]),
         "rpd_reserve": (i32, [vp, i32, i32]),
         "rpd_set_debug": (i32, [vp, ctypes.POINTER(RpdDebug)]),
+        "rpd_set_projection": (i32, [vp, i32]),
         "rpd_step": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_step_batched": (i32, [vp, vp, vp, i32, i32, vp, vp, vp, vp, vp]),
         "rpd_step_host": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
@@ -111,6 +117,7 @@ rpd_get_rule = lib.rpd_get_rule
 rpd_set_stream = lib.rpd_set_stream
 rpd_reserve = lib.rpd_reserve
 rpd_set_debug = lib.rpd_set_debug
+rpd_set_projection = lib.rpd_set_projection
 rpd_step = lib.rpd_step
 rpd_step_batched = lib.rpd_step_batched
 rpd_step_host = lib.rpd_step_host
@@ -177,6 +184,13 @@ class Rpd:
         raw = getattr(stream, "cuda_stream", stream)
         _check(rpd_set_stream(self.handle, ctypes.c_void_p(raw) if raw else None))
 
+    def set_projection(self, mode):
+        """Projection of the window layers (App. A.6): "all", "lazy" (two passes) or "auto"
+        (chosen per step on the device); True/False mean "lazy"/"all"."""
+        if isinstance(mode, bool):
+            mode = "lazy" if mode else "all"
+        _check(rpd_set_projection(self.handle, PROJECTION_MODES[mode]))
+
     def reserve(self, B: int, N: int):
         _check(rpd_reserve(self.handle, B, N))
 
@@ -192,14 +206,15 @@ class Rpd:
 
     def step(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
         """One canvas: hidden [K][N][d] bf16, mask [N] uint8 (in/out), out_commit [N] uint8,
-        out_token [N] int32, out_stats int32 tensor of 8 (an rpd_stats), all CUDA."""
+        out_token [N] int32, out_stats int32 tensor of STATS_WORDS (an rpd_stats), all CUDA."""
         N = mask.numel()
         _check(rpd_step(self.handle, _ptr(hidden), _ptr(mask), N, ctypes.c_float(tau),
                         ctypes.c_float(budget), _ptr(out_commit), _ptr(out_token),
                         _ptr(out_stats)))
 
     def step_batched(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
-        """B canvases: hidden [K][B][N][d], mask/out_commit/out_token [B][N], out_stats [B][8];
+        """B canvases: hidden [K][B][N][d], mask/out_commit/out_token [B][N], out_stats
+        [B][STATS_WORDS];
         tau and budget are length-B host sequences."""
         B, N = mask.shape
         ta = (ctypes.c_float * B)(*[float(x) for x in tau])
@@ -226,6 +241,6 @@ class Rpd:
 
 
 def stats_dict(t) -> dict:
-    """Decode one rpd_stats (an int32 tensor/array of 8) into a dict."""
+    """Decode one rpd_stats (an int32 tensor/array of STATS_WORDS) into a dict."""
     vals = [int(x) for x in (t.tolist() if hasattr(t, "tolist") else t)]
     return dict(zip(STATS_FIELDS, vals))

@@ -27,13 +27,71 @@ __device__ __forceinline__ int warp_inclusive_scan(int v, int lane) {
     return v;
 }
 
+// Head tiling for a pass of `rows` projected rows, chosen on the device (no host round-trip).
+// For each tiling (single-CTA tiles of 128 rows on `single_slots` CTAs, or CTA-pair tiles of
+// 256 rows on `pair_slots` pairs) take the vocabulary split count G minimising
+// waves * n-tiles-per-unit (smallest G on ties); estimate the time as the larger of the MMA
+// work of the busiest slot and the head streaming time scaled by the vocabulary share of the
+// largest split, in single-tile units; keep the cheaper tiling.  Called by every thread of
+// a one-CTA kernel; the result is valid in thread 0.
+__device__ float choose_head_tiling(long long rows, int num_n, int max_splits, int single_slots,
+                                    int pair_slots, float hbm_tiles, int &mode, int &splits) {
+    __shared__ unsigned long long best1, best2;
+    const int tid = threadIdx.x;
+    const int gmax = min(num_n, max_splits);
+    const long long m1 = (rows + kTileM - 1) / kTileM;
+    const long long m2 = (rows + kPairTileM - 1) / kPairTileM;
+    if (tid == 0) best1 = best2 = ~0ull;
+    __syncthreads();
+    unsigned long long key1 = ~0ull, key2 = ~0ull;
+    if (m1 > 0) {
+        for (int g = tid + 1; g <= gmax; g += blockDim.x) {
+            const long long per = (num_n + g - 1) / g;
+            const long long w1 = (m1 * g + single_slots - 1) / single_slots;
+            const unsigned long long k1 = (static_cast<unsigned long long>(w1 * per) << 20) | g;
+            key1 = k1 < key1 ? k1 : key1;
+            if (pair_slots > 0) {
+                const long long w2 = (m2 * g + pair_slots - 1) / pair_slots;
+                const unsigned long long k2 = (static_cast<unsigned long long>(w2 * per) << 20) | g;
+                key2 = k2 < key2 ? k2 : key2;
+            }
+        }
+        atomicMin(&best1, key1);
+        atomicMin(&best2, key2);
+    }
+    __syncthreads();
+    mode = 1;
+    splits = 1;
+    float est = 0.f;
+    if (tid == 0 && m1 > 0) {
+        const int g1 = static_cast<int>(best1 & 0xFFFFFull);
+        const float per1 = static_cast<float>((num_n + g1 - 1) / g1);
+        const float est1 = fmaxf(static_cast<float>(best1 >> 20), hbm_tiles * per1 * g1 / num_n);
+        splits = g1;
+        est = est1;
+        if (pair_slots > 0 && best2 != ~0ull) {
+            const int g2 = static_cast<int>(best2 & 0xFFFFFull);
+            const float per2 = static_cast<float>((num_n + g2 - 1) / g2);
+            const float est2 = fmaxf(kPairTileCost * static_cast<float>(best2 >> 20),
+                                     hbm_tiles * per2 * g2 / num_n);
+            if (est2 < est1) {
+                mode = 2;
+                splits = g2;
+                est = est2;
+            }
+        }
+    }
+    __syncthreads();  // the shared keys may be reused by the next call
+    return est;  // estimated pass time in single-tile units (valid in thread 0)
+}
+
 __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p) {
     __shared__ int warp_sum[32];
     __shared__ unsigned long long best_split;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int block_lo[kMaxBatch];  // RPD-block: first position of each canvas's active block
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
-    pdl_trigger();
     const int total = p.B * p.N;
     if (p.block > 0) {
         for (int b = tid; b < p.B; b += kCompactThreads) block_lo[b] = p.N;
@@ -88,62 +146,103 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
         __syncthreads();
     }
 
-    // Head tiling for this step, chosen from the live row count R = K * NMT (no host
-    // round-trip).  For each tiling (single-CTA tiles of 128 rows on `single_slots` CTAs, or
-    // CTA-pair tiles of 256 rows on `pair_slots` pairs) pick the vocabulary split count G
-    // minimising waves * n-tiles-per-unit (smallest G on ties); estimate the time as the
-    // larger of the MMA work of the busiest slot and the head streaming time (scaled by the
-    // vocabulary share of the largest split), in single-tile units; keep the cheaper one.
-    const long long nm_rows = static_cast<long long>(p.K) * carry;
-    const int gmax = min(p.num_n_tiles, p.max_splits);
-    unsigned long long key1 = ~0ull, key2 = ~0ull;
-    const long long m1 = (nm_rows + kTileM - 1) / kTileM;
-    const long long m2 = (nm_rows + kPairTileM - 1) / kPairTileM;
-    if (tid == 0) best_split = ~0ull;
-    __shared__ unsigned long long best_pair;
-    if (tid == 0) best_pair = ~0ull;
-    __syncthreads();
-    if (m1 > 0) {
-        for (int g = tid + 1; g <= gmax; g += kCompactThreads) {
-            const long long per = (p.num_n_tiles + g - 1) / g;
-            const long long w1 = (m1 * g + p.single_slots - 1) / p.single_slots;
-            const unsigned long long k1 = (static_cast<unsigned long long>(w1 * per) << 20) | g;
-            key1 = k1 < key1 ? k1 : key1;
-            if (p.pair_slots > 0) {
-                const long long w2 = (m2 * g + p.pair_slots - 1) / p.pair_slots;
-                const unsigned long long k2 = (static_cast<unsigned long long>(w2 * per) << 20) | g;
-                key2 = k2 < key2 ? k2 : key2;
-            }
-        }
-        atomicMin(&best_split, key1);
-        atomicMin(&best_pair, key2);
+    // First pass: every window layer of the scored positions, or only the final layer (lazy).
+    // Automatic choice: lazy when its two passes (the final layer of every position, then
+    // the earlier layers of an assumed band fraction) are estimated cheaper than one pass
+    // over all layers.
+    __shared__ int lazy_on;
+    const long long all_rows = static_cast<long long>(p.K) * carry;
+    if (p.lazy == 2 && p.K > 1) {
+        int m_, s_;
+        const float e_all = choose_head_tiling(all_rows, p.num_n_tiles, p.max_splits,
+                                               p.single_slots, p.pair_slots, p.hbm_tiles, m_, s_);
+        const float e_fin = choose_head_tiling(carry, p.num_n_tiles, p.max_splits, p.single_slots,
+                                               p.pair_slots, p.hbm_tiles, m_, s_);
+        const long long guess = static_cast<long long>(kLazyBandGuess * (p.K - 1) * carry);
+        const float e_band = choose_head_tiling(guess, p.num_n_tiles, p.max_splits,
+                                                p.single_slots, p.pair_slots, p.hbm_tiles, m_, s_);
+        if (tid == 0) lazy_on = (e_fin + e_band < e_all) ? 1 : 0;
+    } else if (tid == 0) {
+        lazy_on = (p.lazy == 1 && p.K > 1) ? 1 : 0;
     }
     __syncthreads();
+    const long long rows = lazy_on ? static_cast<long long>(carry) : all_rows;
+    int mode, splits;
+    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.single_slots, p.pair_slots,
+                       p.hbm_tiles, mode, splits);
     if (tid == 0) {
-        int mode = 1, splits = 1;
-        if (m1 > 0) {
-            const int g1 = static_cast<int>(best_split & 0xFFFFFull);
-            const float per1 = static_cast<float>((p.num_n_tiles + g1 - 1) / g1);
-            const float est1 = fmaxf(static_cast<float>(best_split >> 20),
-                                     p.hbm_tiles * per1 * g1 / p.num_n_tiles);
-            splits = g1;
-            if (p.pair_slots > 0 && best_pair != ~0ull) {
-                const int g2 = static_cast<int>(best_pair & 0xFFFFFull);
-                const float per2 = static_cast<float>((p.num_n_tiles + g2 - 1) / g2);
-                const float est2 = fmaxf(kPairTileCost * static_cast<float>(best_pair >> 20),
-                                         p.hbm_tiles * per2 * g2 / p.num_n_tiles);
-                if (est2 < est1) {
-                    mode = 2;
-                    splits = g2;
-                }
-            }
-        }
         p.canvas_off[p.B] = carry;
         p.meta[kMetaMasked] = carry;
-        p.meta[kMetaRows] = static_cast<int>(nm_rows);
+        p.meta[kMetaRows] = static_cast<int>(rows);
         p.meta[kMetaStatus] = RPD_OK;
         p.meta[kMetaSplits] = splits;
         p.meta[kMetaHeadMode] = mode;
+        p.meta[kMetaSel] = carry;
+        p.meta[kMetaLayer0] = lazy_on ? p.K - 1 : 0;
+        p.meta[kMetaRowsTotal] = static_cast<int>(rows);
+        p.meta[kMetaLazy] = lazy_on;
+    }
+}
+
+// Lazy projection, second pass: compact the positions whose final-layer confidence lies in
+// their canvas's stability band (theta_c <= c < tau; Eq. 5 consults S_i only there) and set
+// the pass up over their K-1 earlier window layers.
+__global__ void __launch_bounds__(kCompactThreads, 1) k_band(BandParams p) {
+    __shared__ int warp_sum[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
+    pdl_wait();
+    const int nmt = p.meta[kMetaMasked];
+    const bool lazy_on = p.meta[kMetaLazy] != 0;  // else the first pass covered every layer
+    const float *final_p = p.row_pmax + static_cast<size_t>(p.K - 1) * nmt;
+    int carry = 0;
+    for (int base = 0; lazy_on && base < nmt; base += kCompactThreads * kCompactItems) {
+        const int q0 = base + tid * kCompactItems;
+        int f[kCompactItems];
+        int cnt = 0;
+#pragma unroll
+        for (int j = 0; j < kCompactItems; ++j) {
+            const int q = q0 + j;
+            f[j] = 0;
+            if (lazy_on && q < nmt && p.K > 1) {
+                const float c = final_p[q];
+                const int b = p.pos_of_q[q] / p.N;
+                f[j] = (c >= p.theta_c && c < p.tau[b]) ? 1 : 0;
+            }
+            cnt += f[j];
+        }
+        const int incl = warp_inclusive_scan(cnt, lane);
+        if (lane == 31) warp_sum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            const int v = warp_sum[lane];
+            const int vi = warp_inclusive_scan(v, lane);
+            warp_sum[lane] = vi - v;
+        }
+        __syncthreads();
+        int excl = carry + warp_sum[warp] + incl - cnt;
+#pragma unroll
+        for (int j = 0; j < kCompactItems; ++j) {
+            if (f[j]) p.sel_q[excl] = q0 + j;
+            excl += f[j];
+        }
+        __syncthreads();
+        if (tid == kCompactThreads - 1) warp_sum[0] = excl;
+        __syncthreads();
+        carry = warp_sum[0];
+        __syncthreads();
+    }
+    const long long rows = static_cast<long long>(p.K - 1) * carry;
+    int mode, splits;
+    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.single_slots, p.pair_slots,
+                       p.hbm_tiles, mode, splits);
+    if (tid == 0) {
+        p.meta[kMetaRows] = static_cast<int>(rows);
+        p.meta[kMetaSplits] = splits;
+        p.meta[kMetaHeadMode] = mode;
+        p.meta[kMetaSel] = carry;
+        p.meta[kMetaLayer0] = 0;
+        p.meta[kMetaRowsTotal] += static_cast<int>(rows);
     }
 }
 
@@ -159,15 +258,18 @@ __global__ void __launch_bounds__(kNormThreads) k_gather_norm(NormParams p) {
     const int nvec = p.d >> 3;  // 8 bf16 per 16-byte vector
     const uint4 *__restrict__ gvec = reinterpret_cast<const uint4 *>(p.gain);
     for (int v = threadIdx.x; v < nvec; v += blockDim.x) g_smem[v] = __ldg(gvec + v);
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
-    pdl_trigger();
     __syncthreads();
-    const int nmt = p.meta[kMetaMasked];
+    const int sel = p.meta[kMetaSel];
+    const int layer0 = p.meta[kMetaLayer0];
     const int rows = p.meta[kMetaRows];
     for (int r = blockIdx.x * warps_per_cta + (threadIdx.x >> 5); r < rows;
          r += gridDim.x * warps_per_cta) {
-        const int k = r / nmt;
-        const int q = r - k * nmt;
+        const int kr = r / sel;
+        const int sr = r - kr * sel;
+        const int k = layer0 + kr;
+        const int q = p.sel_list ? p.sel_list[sr] : sr;
         const int pos = p.pos_of_q[q];
         const uint4 *__restrict__ src =
             reinterpret_cast<const uint4 *>(p.hidden + (static_cast<size_t>(k) * p.BN + pos) * p.d);
@@ -211,6 +313,10 @@ __global__ void __launch_bounds__(kNormThreads) k_gather_norm(NormParams p) {
 
 cudaError_t launch_compact(const CompactParams &p, cudaStream_t s) {
     return launch_pdl(k_compact, dim3(1), dim3(kCompactThreads), 0, s, p);
+}
+
+cudaError_t launch_band(const BandParams &p, cudaStream_t s) {
+    return launch_pdl(k_band, dim3(1), dim3(kCompactThreads), 0, s, p);
 }
 
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s) {

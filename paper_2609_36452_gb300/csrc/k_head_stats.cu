@@ -80,8 +80,9 @@ __device__ __forceinline__ void fold_chunk(const float (&v)[32], float scale, in
 __global__ void __launch_bounds__(kHeadThreads, 1)
     k_head_stats(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW,
                  HeadParams p) {
-    pdl_wait();  // row count, tiling, u and inv_rms come from the preceding kernels
-    if (p.meta[kMetaHeadMode] != 1) return;  // the CTA-pair tiling runs this step
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
+    pdl_wait();     // row count, tiling, u and inv_rms come from the preceding kernels
+    if (p.meta[kMetaHeadMode] != 1 || p.meta[kMetaRows] == 0) return;  // pair tiling, or nothing to do
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -261,7 +262,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     }
 
     __syncwarp();
-    pdl_trigger();  // the merge kernel may launch once every CTA is past its main loop
     tc_fence_before_sync();
     __syncthreads();
     tc_fence_after_sync();
@@ -288,8 +288,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 __global__ void __launch_bounds__(kHeadThreads, 1)
     k_head_stats_pair(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW,
                       HeadParams p) {
-    pdl_wait();  // row count, tiling, u and inv_rms come from the preceding kernels
-    if (p.meta[kMetaHeadMode] != 2) return;  // the single-CTA tiling runs this step
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
+    pdl_wait();     // row count, tiling, u and inv_rms come from the preceding kernels
+    if (p.meta[kMetaHeadMode] != 2 || p.meta[kMetaRows] == 0) return;  // single tiling, or nothing
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -481,7 +482,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     }
 
     __syncwarp();
-    pdl_trigger();
     tc_fence_before_sync();
     __syncthreads();
     cluster_sync();  // no signal may still be in flight to a CTA that is about to exit

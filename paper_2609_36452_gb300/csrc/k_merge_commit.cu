@@ -50,13 +50,20 @@ __device__ __forceinline__ Stat merge2(const Stat &x, const Stat &y) {
 }
 
 __global__ void __launch_bounds__(256) k_merge(MergeParams p) {
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
-    pdl_trigger();
     const int rows = p.meta[kMetaRows];
     const int splits = p.meta[kMetaSplits];
+    const int nmt = p.meta[kMetaMasked];
+    const int sel = p.meta[kMetaSel];
+    const int layer0 = p.meta[kMetaLayer0];
     const int lane = threadIdx.x & 31;
     const int wpc = blockDim.x >> 5;
     for (int r = blockIdx.x * wpc + (threadIdx.x >> 5); r < rows; r += gridDim.x * wpc) {
+        // this pass's row r is layer layer0 + r / sel of compact position sel_list[r % sel]
+        const int kr = r / sel;
+        const int sr = r - kr * sel;
+        const size_t out = static_cast<size_t>(layer0 + kr) * nmt + (p.sel_list ? p.sel_list[sr] : sr);
         Stat acc{-INFINITY, 0.f, 0.f, 0x7fffffff};
         const float4 *row = p.partials + static_cast<size_t>(r) * p.max_splits;
         for (int g = lane; g < splits; g += 32) {
@@ -74,9 +81,9 @@ __global__ void __launch_bounds__(256) k_merge(MergeParams p) {
             acc = (lane & o) ? merge2(other, acc) : merge2(acc, other);
         }
         if (lane == 0) {
-            p.row_arg[r] = acc.a;
-            p.row_pmax[r] = 1.0f / acc.s;
-            p.row_H[r] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
+            p.row_arg[out] = acc.a;
+            p.row_pmax[out] = 1.0f / acc.s;
+            p.row_H[out] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
         }
     }
 }
@@ -157,8 +164,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     __shared__ int first_reject;
     __shared__ unsigned long long best_fb;
 
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
-    pdl_trigger();
     const int b = blockIdx.x;
     const int N = p.N;
     const int nmt = p.meta[kMetaMasked];
@@ -168,6 +175,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     const int i0 = threadIdx.x * items;
     uint8_t *mask = p.mask + static_cast<size_t>(b) * N;
     const bool dbg_layers = p.dbg.layer_argmax || p.dbg.layer_pmax;
+    const bool lazy_on = p.meta[kMetaLazy] != 0;  // earlier layers exist only in the band
 
     bool masked[kMaxItems], cand[kMaxItems], high[kMaxItems];
     int y[kMaxItems];
@@ -195,6 +203,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
             // Backward over the window, a batch of layers at a time (loads issued together).
             float peak = 0.f;
             bool run = true;
+            bool projected = true;  // lazy projection: earlier layers exist only in the band
             for (int k_hi = K; k_hi > 0; k_hi -= kLayerBatch) {
                 if (!run && !dbg_layers) break;  // persistence settled; debug wants every layer
                 int a_b[kLayerBatch];
@@ -217,6 +226,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
                         conf[j] = p_b[t];
                         peak = p_b[t];
                         ki = 1;
+                        if (lazy_on && !(conf[j] >= p.theta_c && conf[j] < tau)) {
+                            projected = false;  // outside the band: K_i, r_i not needed
+                            run = false;
+                        }
+                    } else if (!projected) {
+                        a_b[t] = -1;
+                        p_b[t] = 0.f;
                     } else if (run) {
                         if (a_b[t] != y[j]) {
                             run = false;
@@ -237,6 +253,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
             s = static_cast<float>(min(ki, p.k_max)) - p.w * r;
             high[j] = conf[j] >= tau;
             cand[j] = high[j] || (conf[j] >= p.theta_c && conf[j] < tau && s >= p.theta_s);
+            if (!projected) {  // reported as not evaluated
+                ki = 0;
+                r = 0.f;
+                s = 0.f;
+            }
             ++local.m;
             n_cand += cand[j];
             if (!cand[j]) local.q += H[j];
@@ -333,6 +354,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
         st.fallback_used = fb_pos >= 0 ? 1 : 0;
         st.fallback_pos = fb_pos;
         st.status = p.meta[kMetaStatus];
+        st.n_rows = p.meta[kMetaRowsTotal];
         p.out_stats[b] = st;
     }
 }

@@ -22,7 +22,9 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 // may start while its predecessor in the stream is still running.  pdl_wait() blocks until
 // the predecessor grid has completed and its memory is visible (a no-op otherwise); every
 // kernel calls it before touching global memory that a predecessor reads or writes.
-// pdl_trigger() lets the successor grid launch once every CTA of this grid has triggered.
+// pdl_trigger() lets the successor grid launch once every CTA of this grid has triggered;
+// the kernels trigger on entry, so a successor's CTAs are resident (and blocked in their
+// own pdl_wait) by the time this grid completes.
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 

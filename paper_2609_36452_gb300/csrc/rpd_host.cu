@@ -95,6 +95,8 @@ struct rpd_ctx {
     int32_t *row_arg = nullptr;
     float *row_pmax = nullptr, *row_H = nullptr;
     int32_t *q_of_pos = nullptr, *pos_of_q = nullptr, *canvas_off = nullptr, *meta = nullptr;
+    int32_t *sel_q = nullptr;  // lazy projection: compact indices of the band positions
+    int projection = RPD_PROJECT_ALL;
     CUtensorMap tmU{}, tmW{}, tmW_pair{};
     int pair_grid = 0;   // CTAs of the CTA-pair head kernel (2 x resident pairs; 0 = none)
 
@@ -110,7 +112,7 @@ struct rpd_ctx {
 
     void free_scratch() {
         void *ptrs[] = {u, inv_rms, partials, row_arg, row_pmax, row_H, q_of_pos, pos_of_q,
-                        canvas_off, meta};
+                        canvas_off, meta, sel_q};
         for (void *p : ptrs)
             if (p) cudaFree(p);
         u = nullptr;
@@ -118,7 +120,7 @@ struct rpd_ctx {
         partials = nullptr;
         row_arg = nullptr;
         row_pmax = row_H = nullptr;
-        q_of_pos = pos_of_q = canvas_off = meta = nullptr;
+        q_of_pos = pos_of_q = canvas_off = meta = sel_q = nullptr;
         cap_bn = cap_b = cap_rows = 0;
     }
 };
@@ -151,6 +153,7 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
         {reinterpret_cast<void **>(&c->row_H), static_cast<size_t>(rows) * 4},
         {reinterpret_cast<void **>(&c->q_of_pos), static_cast<size_t>(new_bn) * 4},
         {reinterpret_cast<void **>(&c->pos_of_q), static_cast<size_t>(new_bn) * 4},
+        {reinterpret_cast<void **>(&c->sel_q), static_cast<size_t>(new_bn) * 4},
         {reinterpret_cast<void **>(&c->canvas_off), static_cast<size_t>(new_b + 1) * 4},
         {reinterpret_cast<void **>(&c->meta), kMetaWords * 4},
     };
@@ -246,37 +249,71 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
     const int bn = B * N;
     const int num_n = (c->V + kTileN - 1) / kTileN;
     const int pair_slots = c->pair_grid / 2;
+    const float hbm_tiles = head_stream_in_tiles(c->V, c->d, c->num_sms);
+    // Lazy projection (forced, or chosen on the device per step): a second pass over the band.
+    // It is not launched when even the largest possible row count keeps a single pass cheaper.
+    const bool lazy = c->projection == RPD_PROJECT_LAZY ||
+                      (c->projection == RPD_PROJECT_AUTO && c->K > 1 &&
+                       static_cast<long long>(c->K) * bn > 2LL * kTileM);
     cudaError_t e;
     {
         KernelTimer t(c, 0);
         CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
-                         num_n, c->max_splits, c->num_sms, pair_slots,
-                         head_stream_in_tiles(c->V, c->d, c->num_sms), c->rule.block};
+                         num_n, c->max_splits, c->num_sms, pair_slots, hbm_tiles, c->rule.block,
+                         c->projection == RPD_PROJECT_LAZY ? 1 : (lazy ? 2 : 0)};
         e = launch_compact(cp, c->stream);
-        if (e == cudaSuccess) {
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "compaction launch");
+    // One projection pass: gather + RMSNorm prologue, head statistics, merge.  Rows, layers and
+    // positions of the pass come from the device-side meta words.
+    auto pass = [&](const int32_t *sel_list) -> cudaError_t {
+        cudaError_t err;
+        {
+            KernelTimer t(c, 0);
             NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
-                          static_cast<const __nv_bfloat16 *>(c->g), c->pos_of_q, c->meta, c->u,
-                          c->inv_rms, bn, c->d, c->eps};
-            e = launch_gather_norm(np, c->num_sms * 8, c->stream);
+                          static_cast<const __nv_bfloat16 *>(c->g), c->pos_of_q, sel_list, c->meta,
+                          c->u, c->inv_rms, bn, c->d, c->eps};
+            err = launch_gather_norm(np, c->num_sms * 8, c->stream);
         }
-    }
-    if (e != cudaSuccess) return cuda_fail(e, "gather/norm launch");
-    {
-        KernelTimer t(c, 1);
-        HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits};
-        // Both tilings are launched; each reads the choice k_compact made for this step's row
-        // count and the other returns at once.
-        e = launch_head_stats(c->tmU, c->tmW, hp, c->num_sms, c->stream);
-        if (e == cudaSuccess && pair_slots > 0)
-            e = launch_head_stats_pair(c->tmU, c->tmW_pair, hp, c->pair_grid, c->stream);
-    }
-    if (e != cudaSuccess) return cuda_fail(e, "head statistics launch");
-    {
+        if (err != cudaSuccess) return err;
+        {
+            KernelTimer t(c, 1);
+            HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits};
+            // Both tilings are launched; each reads the choice made on the device for this
+            // pass's row count and the other returns at once.
+            err = launch_head_stats(c->tmU, c->tmW, hp, c->num_sms, c->stream);
+            if (err == cudaSuccess && pair_slots > 0)
+                err = launch_head_stats_pair(c->tmU, c->tmW_pair, hp, c->pair_grid, c->stream);
+        }
+        if (err != cudaSuccess) return err;
         KernelTimer t(c, 2);
-        MergeParams mp{c->partials, c->meta, c->row_arg, c->row_pmax, c->row_H, c->max_splits};
-        e = launch_merge(mp, c->num_sms * 8, c->stream);
+        MergeParams mp{c->partials, sel_list, c->meta, c->row_arg, c->row_pmax, c->row_H,
+                       c->max_splits};
+        return launch_merge(mp, c->num_sms * 8, c->stream);
+    };
+    e = pass(nullptr);
+    if (e == cudaSuccess && lazy) {
+        {
+            KernelTimer t(c, 2);
+            BandParams bp{};
+            bp.meta = c->meta;
+            bp.pos_of_q = c->pos_of_q;
+            bp.row_pmax = c->row_pmax;
+            bp.sel_q = c->sel_q;
+            bp.N = N;
+            bp.K = c->K;
+            bp.theta_c = c->rule.theta_c;
+            bp.num_n_tiles = num_n;
+            bp.max_splits = c->max_splits;
+            bp.single_slots = c->num_sms;
+            bp.pair_slots = pair_slots;
+            bp.hbm_tiles = hbm_tiles;
+            for (int b = 0; b < B; ++b) bp.tau[b] = tau[b];
+            e = launch_band(bp, c->stream);
+        }
+        if (e == cudaSuccess) e = pass(c->sel_q);
     }
-    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+    if (e != cudaSuccess) return cuda_fail(e, "projection launch");
     {
         KernelTimer t(c, 3);
         ScoreParams sp{};
@@ -300,6 +337,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         sp.k_max = c->rule.k_max;
         sp.window = c->rule.window;
         sp.block = c->rule.block;
+        sp.lazy = lazy ? 1 : 0;
         for (int b = 0; b < B; ++b) {
             sp.tau[b] = tau[b];
             sp.budget[b] = budget[b];
@@ -404,6 +442,14 @@ int rpd_reserve(rpd_ctx *c, int B, int N) {
     if (B < 1 || B > kMaxBatch || N < 1 || N > kMaxCanvas)
         return fail(RPD_ERR_INVALID_ARGUMENT, "reserve: B in [1,%d], N in [1,%d]", kMaxBatch, kMaxCanvas);
     return ensure_scratch(c, B, N);
+}
+
+int rpd_set_projection(rpd_ctx *c, int mode) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (mode != RPD_PROJECT_ALL && mode != RPD_PROJECT_LAZY && mode != RPD_PROJECT_AUTO)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "unknown projection mode %d", mode);
+    c->projection = mode;
+    return RPD_OK;
 }
 
 int rpd_set_debug(rpd_ctx *c, const rpd_debug *dbg) {

@@ -40,7 +40,11 @@ enum MetaIndex : int {
     kMetaStatus = 2,   // RPD_OK or RPD_ERR_TIMEOUT, latched by kernels
     kMetaSplits = 3,   // vocabulary splits G chosen for the head kernel
     kMetaHeadMode = 4, // 1: single-CTA head tiles, 2: CTA-pair head tiles
-    kMetaWords = 8
+    kMetaSel = 5,      // positions projected by the current pass
+    kMetaLayer0 = 6,   // first window layer of the current pass (rows are layer-major)
+    kMetaRowsTotal = 7,// rows projected by all passes of this step
+    kMetaLazy = 8,     // 1 when this step projects lazily (two passes)
+    kMetaWords = 16
 };
 
 struct CompactParams {
@@ -56,6 +60,26 @@ struct CompactParams {
     int pair_slots;       // CTA pairs of the pair head kernel (0: pair tiles unavailable)
     float hbm_tiles;      // time to stream the head once, in single-CTA tile times
     int block;            // 0: every masked position; > 0: only each canvas's active block
+    int lazy;             // 0: all window layers; 1: lazy; 2: lazy when it is estimated cheaper
+};
+
+// Band fraction assumed when the device weighs lazy against full projection before the
+// first pass (the real band is known only after it).
+constexpr float kLazyBandGuess = 0.25f;
+
+// Second pass of lazy projection: selects the positions whose final confidence lies in the
+// stability band theta_c <= c < tau of their canvas and sets up the pass over their earlier
+// window layers (tiling, split count, row mapping).
+struct BandParams {
+    int32_t *meta;
+    const int32_t *pos_of_q;   // [NMT] flat position b*N+i of compact index q
+    const float *row_pmax;     // final-layer probabilities at (K-1)*NMT + q
+    int32_t *sel_q;            // out: compact indices of the band positions
+    int N, K;
+    float theta_c;
+    int num_n_tiles, max_splits, single_slots, pair_slots;
+    float hbm_tiles;
+    float tau[kMaxBatch];
 };
 
 // Relative cost of a CTA-pair tile (256 rows on two SMs) against a single-CTA tile (128 rows
@@ -66,10 +90,14 @@ constexpr float kPairTileCost = 0.88f;
 constexpr double kSingleTileFlopsPerSm = 1.1e13;
 constexpr double kHeadStreamBytesPerSec = 6.5e12;
 
+// Row r of a projection pass: layer k = meta[kMetaLayer0] + r / S and position
+// q = sel[r % S] (sel = the pass's list of compact indices, or the identity when null),
+// S = meta[kMetaSel]; its statistics land at k * NMT + q.
 struct NormParams {
     const __nv_bfloat16 *hidden;  // [K][B*N][d]
     const __nv_bfloat16 *gain;    // [d]
     const int32_t *pos_of_q;
+    const int32_t *sel_list;      // null: every compact position
     const int32_t *meta;
     __nv_bfloat16 *u;             // [rows][d] compact head operand bf16(g*h)
     float *inv_rms;               // [rows]
@@ -94,6 +122,7 @@ inline float head_stream_in_tiles(int V, int d, int num_sms) {
 
 struct MergeParams {
     const float4 *partials;
+    const int32_t *sel_list;  // as in NormParams
     const int32_t *meta;
     int32_t *row_arg;   // [rows]
     float *row_pmax;    // [rows]
@@ -117,6 +146,7 @@ struct ScoreParams {
     float theta_c, theta_s, w;
     int k_max, window;
     int block;                  // 0: full RPD; > 0: RPD-block (no budget, in-block fallback)
+    int lazy;                   // 1: earlier window layers exist only for band positions
     float tau[kMaxBatch];
     float budget[kMaxBatch];
 };
@@ -153,6 +183,7 @@ cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tm
 // Largest number of CTA pairs of the pair kernel that can be resident at once.
 int head_stats_pair_max_clusters();
 cudaError_t launch_merge(const MergeParams &p, int grid, cudaStream_t s);
+cudaError_t launch_band(const BandParams &p, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
 
 }  // namespace rpd

@@ -202,13 +202,13 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     if (e == cudaSuccess) {
         CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n, splits,
                          dev->num_sms, pair_slots, head_stream_in_tiles(V, d, dev->num_sms),
-                         rule.block};
+                         rule.block, 0};
         e = launch_compact(cp, stream);
     }
     if (e == cudaSuccess) {
         NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
-                      static_cast<const __nv_bfloat16 *>(g_norm), pos_of_q, meta, u, inv_rms, N, d,
-                      eps};
+                      static_cast<const __nv_bfloat16 *>(g_norm), pos_of_q, nullptr, meta, u,
+                      inv_rms, N, d, eps};
         e = launch_gather_norm(np, dev->num_sms * 8, stream);
     }
     if (e == cudaSuccess) {
@@ -218,7 +218,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
             e = launch_head_stats_pair(tmU, tmW_pair, hp, dev->pair_grid, stream);
     }
     if (e == cudaSuccess) {
-        MergeParams mp{partials, meta, row_arg, row_pmax, row_H, splits};
+        MergeParams mp{partials, nullptr, meta, row_arg, row_pmax, row_H, splits};
         e = launch_merge(mp, dev->num_sms * 8, stream);
     }
     if (e == cudaSuccess) {

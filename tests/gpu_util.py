@@ -38,7 +38,7 @@ class GpuRunner:
         out = dict(
             commit=torch.full((B, N), 7, dtype=torch.uint8, device=dev),
             token=torch.full((B, N), -5, dtype=torch.int32, device=dev),
-            stats=torch.full((B, 8), -9, dtype=torch.int32, device=dev),
+            stats=torch.full((B, self.rpd.STATS_WORDS), -9, dtype=torch.int32, device=dev),
             conf=torch.full((B, N), -1.0, device=dev),
             entropy=torch.full((B, N), -1.0, device=dev),
             persist=torch.full((B, N), -1, dtype=torch.int32, device=dev),

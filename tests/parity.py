@@ -114,10 +114,24 @@ def near_threshold_positions(ref: O.StepResult):
     return out
 
 
-def compare_step(ref: O.StepResult, got: dict, check_scores: bool = True) -> ParityReport:
+def lazy_band(ref: O.StepResult):
+    """Positions whose earlier window layers a lazy step projects (theta_c <= c < tau), and
+    those within DELTA of the band's edges (either side may be taken)."""
+    p = ref.params
+    c = ref.conf
+    m = ref.masked & np.isfinite(c)
+    band = m & (c >= p["theta_c"]) & (c < p["tau"])
+    edge = m & ((np.abs(c - p["theta_c"]) < DELTA) | (np.abs(c - p["tau"]) < DELTA))
+    return band, edge
+
+
+def compare_step(ref: O.StepResult, got: dict, check_scores: bool = True,
+                 lazy: bool = False) -> ParityReport:
     """``got`` holds numpy arrays for one canvas: commit, token (after the step; only
     committed positions are compared), new_mask, stats (dict) and optionally conf,
-    entropy, persist, drop, candidate, layer_argmax [K][N], layer_pmax [K][N]."""
+    entropy, persist, drop, candidate, layer_argmax [K][N], layer_pmax [K][N].
+    ``lazy``: the step projected earlier window layers only for band positions, so those
+    layers (and K_i, r_i) are compared there only."""
     rep = ParityReport()
     m = ref.masked
     rep.n_masked = int(m.sum())
@@ -125,6 +139,7 @@ def compare_step(ref: O.StepResult, got: dict, check_scores: bool = True) -> Par
     rep.near_threshold = free
     free_set = set(free)
     K = ref.layer_argmax.shape[0]
+    band, edge = lazy_band(ref) if lazy else (np.ones_like(m), np.zeros_like(m))
 
     if check_scores and "conf" in got:
         idx = np.nonzero(m)[0]
@@ -137,6 +152,8 @@ def compare_step(ref: O.StepResult, got: dict, check_scores: bool = True) -> Par
             la, lp = got["layer_argmax"], got["layer_pmax"]
             for i in idx:
                 for k in range(K):
+                    if k < K - 1 and (not band[i] or edge[i]):
+                        continue  # lazy: not projected outside the band
                     if ref.layer_gap[k, i] < DELTA:
                         rep.argmax_exempt += 1
                         continue
@@ -145,7 +162,7 @@ def compare_step(ref: O.StepResult, got: dict, check_scores: bool = True) -> Par
             assert rep.max_dpmax < PROB_TOL, f"layer max probability off by {rep.max_dpmax}"
         if "persist" in got:
             for i in idx:
-                if np.nanmin(ref.layer_gap[:, i]) < DELTA:
+                if np.nanmin(ref.layer_gap[:, i]) < DELTA or not band[i] or edge[i]:
                     continue
                 assert got["persist"][i] == ref.persist[i], (i, got["persist"][i], ref.persist[i])
                 assert abs(got["drop"][i] - ref.drop[i]) < 2 * PROB_TOL, (i, got["drop"][i], ref.drop[i])

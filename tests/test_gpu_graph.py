@@ -31,7 +31,7 @@ def test_step_replays_from_cuda_graph():
     def outputs():
         return (mask0.clone(), torch.zeros(N, dtype=torch.uint8, device=dev),
                 torch.full((N,), -1, dtype=torch.int32, device=dev),
-                torch.zeros(8, dtype=torch.int32, device=dev))
+                torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev))
 
     # eager reference (also configures the kernels before capture)
     ctx.set_stream(torch.cuda.current_stream(dev))

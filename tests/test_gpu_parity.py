@@ -21,6 +21,11 @@ if not torch.cuda.is_available():  # collected on CPU machines, never run there
     pytest.skip("needs a CUDA GPU", allow_module_level=True)
 
 
+def rpd_mod():
+    import paper_2609_36452_gb300 as rpd
+    return rpd
+
+
 def oracle_step(case, hidden=None, mask=None, tau=None, budget=None, rule=None):
     hidden = case["hidden"] if hidden is None else hidden
     mask = case["mask"] if mask is None else mask
@@ -184,7 +189,7 @@ def test_host_entry_point_matches_device():
         mask = case["mask"].clone().pin_memory()
         commit = torch.zeros(64, dtype=torch.uint8).pin_memory()
         token = torch.full((64,), -5, dtype=torch.int32).pin_memory()
-        stats = torch.zeros(8, dtype=torch.int32).pin_memory()
+        stats = torch.zeros(rpd_mod().STATS_WORDS, dtype=torch.int32).pin_memory()
         runner.ctx.set_debug()
         runner.ctx.step_host(hid, mask, 0.9, 1.0, commit, token, stats)
         assert np.array_equal(commit.numpy(), dev["commit"])
@@ -220,7 +225,7 @@ def test_invalid_arguments_on_gpu():
     m = torch.ones(8, dtype=torch.uint8, device=dev)
     c = torch.zeros(8, dtype=torch.uint8, device=dev)
     t = torch.zeros(8, dtype=torch.int32, device=dev)
-    s = torch.zeros(8, dtype=torch.int32, device=dev)
+    s = torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev)
     with pytest.raises(rpd.RpdError) as e:
         ctx.step(h, m, 0.9, 1.0, c, t, s)
     assert e.value.code == rpd.RPD_ERR_NO_HEAD
@@ -325,3 +330,93 @@ def test_rpd_block_llada_first_step_full(llada_head):
                            case["eps"], case["tau"], rule, block=32)
     rep = compare_block_step(ref, got)
     print(rep, got["stats"])
+
+
+# ----------------------------------------------------------------------------- lazy projection
+
+def run_lazy_and_eager(case, rule=None, tau=None, budget=None):
+    outs = {}
+    for lazy in (False, True):
+        runner = GpuRunner(case["W"], case["g"], case["K"], case["eps"],
+                           rule=case["rule"] if rule is None else rule)
+        runner.ctx.set_projection(lazy)
+        try:
+            outs[lazy] = runner.step(case["hidden"], case["mask"], case["tau"] if tau is None else tau,
+                                     case["budget"] if budget is None else budget)
+        finally:
+            runner.close()
+    return outs[False], outs[True]
+
+
+def check_lazy(case, eager, lazy, ref, K):
+    rep = compare_step(ref, lazy, lazy=True)
+    assert np.array_equal(lazy["commit"], eager["commit"])
+    assert np.array_equal(lazy["new_mask"], eager["new_mask"])
+    sel = lazy["commit"] == 1
+    assert np.array_equal(lazy["token"][sel], eager["token"][sel])
+    m = case["mask"].numpy().astype(bool)
+    c = lazy["conf"]
+    p = ref.params
+    # the band test in the same precision as the kernel (fp32 confidences and thresholds)
+    n_band = int(np.sum(m & (c >= np.float32(p["theta_c"])) & (c < np.float32(p["tau"]))))
+    assert eager["stats"]["n_rows"] == K * int(m.sum())
+    assert lazy["stats"]["n_rows"] == int(m.sum()) + (K - 1) * n_band
+    return rep, n_band
+
+
+@pytest.mark.parametrize("seed", [201, 202, 203])
+def test_lazy_projection_small(seed):
+    case = small_case(seed, K=5, N=160, a=torch.ones(5), flip=0.15, mask_frac=0.8)
+    rule = dict(O.RULES["llada"], theta_s=3.0)
+    eager, lazy = run_lazy_and_eager(case, rule=rule)
+    ref = oracle_step(case, rule=rule)
+    rep, n_band = check_lazy(case, eager, lazy, ref, case["K"])
+    print(rep, "band", n_band, lazy["stats"])
+
+
+def test_lazy_projection_empty_band():
+    """No confidence in [theta_c, tau): the second pass has no rows and the head is streamed
+    once."""
+    case = small_case(205, K=4, N=64, w_std=0.02, sigma=1.0)   # every confidence ~ 1/V
+    eager, lazy = run_lazy_and_eager(case)
+    ref = oracle_step(case)
+    rep, n_band = check_lazy(case, eager, lazy, ref, case["K"])
+    assert n_band == 0 and lazy["stats"]["n_rows"] == 64
+
+
+def test_lazy_projection_llada_full(llada_head):
+    W, g = llada_head
+    case = WL.llada_first_step(seed=2, W=W, g=g)
+    eager, lazy = run_lazy_and_eager(case)
+    ref = oracle_step(case)
+    rep, n_band = check_lazy(case, eager, lazy, ref, case["K"])
+    print(rep, "band", n_band, lazy["stats"])
+
+
+def test_auto_projection_picks_per_step(llada_head):
+    """Automatic projection: lazy at the LLaDA first step (1024 rows: bound by the tensor
+    cores), every layer when 5 positions remain (bound by streaming the head); commits equal
+    the all-layer step either way."""
+    W, g = llada_head
+    case = WL.llada_first_step(seed=2, W=W, g=g)
+    tail = case["mask"].clone()
+    tail[:-5] = 0
+    for mask, expect_lazy in ((case["mask"], True), (tail, False)):
+        outs = {}
+        for mode in ("all", "auto"):
+            runner = GpuRunner(W, g, case["K"], case["eps"], rule="llada")
+            runner.ctx.set_projection(mode)
+            try:
+                outs[mode] = runner.step(case["hidden"], mask, case["tau"], case["budget"])
+            finally:
+                runner.close()
+        a, b = outs["all"], outs["auto"]
+        assert np.array_equal(a["commit"], b["commit"]) and np.array_equal(a["new_mask"], b["new_mask"])
+        sel = a["commit"] == 1
+        assert np.array_equal(a["token"][sel], b["token"][sel])
+        nm = int(mask.sum())
+        assert a["stats"]["n_rows"] == case["K"] * nm
+        if expect_lazy:
+            assert b["stats"]["n_rows"] < case["K"] * nm
+        else:
+            assert b["stats"]["n_rows"] == case["K"] * nm

@@ -399,3 +399,21 @@ def test_full_step_no_mask():
     h, mask, gain, W = _tiny_inputs(23)
     r = O.rpd_step(h, np.zeros_like(mask), gain, W, 1e-6, 0.9, 1.0, "llada")
     assert r.commit.sum() == 0 and r.fallback_pos == -1
+
+
+def test_only_band_positions_need_earlier_layers():
+    """Eq. 5: outside theta_c <= c < theta_h a position's candidacy does not depend on S_i,
+    so the earlier window layers of such positions can be replaced by anything without
+    changing the commit set (what lazy projection relies on, App. A.6)."""
+    rng = np.random.default_rng(31)
+    for seed in range(10):
+        h, mask, gain, W = _tiny_inputs(200 + seed, K=4, N=30)
+        r = O.rpd_step(h, mask, gain, W, 1e-6, 0.9, 1.0, "llada")
+        band = r.masked & (r.conf >= 0.6) & (r.conf < 0.9)
+        A = r.layer_argmax.copy()
+        P = r.p_of_y.copy()
+        for i in np.nonzero(r.masked & ~band)[0]:
+            A[:-1, i] = rng.integers(0, 64, size=A.shape[0] - 1)
+            P[:-1, i] = rng.random(A.shape[0] - 1)
+        commit, cand, acc, fb = O.step_from_scores(r.masked, A, P, r.H, 0.9, 1.0, "llada")
+        assert np.array_equal(commit, r.commit) and np.array_equal(cand, r.cand)

@@ -43,7 +43,7 @@ def make_case(seed, K, N, d, V, mask_frac):
 def outputs(N):
     return (torch.full((N,), 7, dtype=torch.uint8, device=DEV),
             torch.full((N,), -5, dtype=torch.int32, device=DEV),
-            torch.full((8,), -9, dtype=torch.int32, device=DEV))
+            torch.full((rpd.STATS_WORDS,), -9, dtype=torch.int32, device=DEV))
 
 
 def run_context(case, tau, budget):
