@@ -6,11 +6,13 @@
 //   q = 0..NMT-1 (canvas-major, then position), per-canvas offsets, the projected row
 //   count R = K*NMT and the vocabulary split count the head kernel will use.  Nothing
 //   goes back to the host: later kernels read these words from device memory.
-// k_gather_norm (grid-stride, one warp per row): row r = k*NMT + q reads hidden[k][pos(q)],
-//   writes the head operand u[r] = bf16_rne(g * h) (exact product, one rounding) and
+// k_gather_norm (grid-stride, one warp per row): row r of a projection pass (layer k and
+//   compact position q from the pass's meta words) reads hidden[k][pos(q)], writes the head
+//   operand u[r] = bf16_rne(g * h) (exact product, one rounding) and
 //   inv_rms[r] = (mean(h^2) + eps)^(-1/2); the RMS factor is applied after the contraction.
 #include "ptx.cuh"
 #include "rpd_internal.h"
+#include "step_common.cuh"
 
 namespace rpd {
 namespace {
@@ -18,76 +20,8 @@ namespace {
 constexpr int kCompactThreads = 1024;
 constexpr int kCompactItems = 4;
 
-__device__ __forceinline__ int warp_inclusive_scan(int v, int lane) {
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        int t = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= o) v += t;
-    }
-    return v;
-}
-
-// Head tiling for a pass of `rows` projected rows, chosen on the device (no host round-trip).
-// For each tiling (single-CTA tiles of 128 rows on `single_slots` CTAs, or CTA-pair tiles of
-// 256 rows on `pair_slots` pairs) take the vocabulary split count G minimising
-// waves * n-tiles-per-unit (smallest G on ties); estimate the time as the larger of the MMA
-// work of the busiest slot and the head streaming time scaled by the vocabulary share of the
-// largest split, in single-tile units; keep the cheaper tiling.  Called by every thread of
-// a one-CTA kernel; the result is valid in thread 0.
-__device__ float choose_head_tiling(long long rows, int num_n, int max_splits, int single_slots,
-                                    int pair_slots, float hbm_tiles, int &mode, int &splits) {
-    __shared__ unsigned long long best1, best2;
-    const int tid = threadIdx.x;
-    const int gmax = min(num_n, max_splits);
-    const long long m1 = (rows + kTileM - 1) / kTileM;
-    const long long m2 = (rows + kPairTileM - 1) / kPairTileM;
-    if (tid == 0) best1 = best2 = ~0ull;
-    __syncthreads();
-    unsigned long long key1 = ~0ull, key2 = ~0ull;
-    if (m1 > 0) {
-        for (int g = tid + 1; g <= gmax; g += blockDim.x) {
-            const long long per = (num_n + g - 1) / g;
-            const long long w1 = (m1 * g + single_slots - 1) / single_slots;
-            const unsigned long long k1 = (static_cast<unsigned long long>(w1 * per) << 20) | g;
-            key1 = k1 < key1 ? k1 : key1;
-            if (pair_slots > 0) {
-                const long long w2 = (m2 * g + pair_slots - 1) / pair_slots;
-                const unsigned long long k2 = (static_cast<unsigned long long>(w2 * per) << 20) | g;
-                key2 = k2 < key2 ? k2 : key2;
-            }
-        }
-        atomicMin(&best1, key1);
-        atomicMin(&best2, key2);
-    }
-    __syncthreads();
-    mode = 1;
-    splits = 1;
-    float est = 0.f;
-    if (tid == 0 && m1 > 0) {
-        const int g1 = static_cast<int>(best1 & 0xFFFFFull);
-        const float per1 = static_cast<float>((num_n + g1 - 1) / g1);
-        const float est1 = fmaxf(static_cast<float>(best1 >> 20), hbm_tiles * per1 * g1 / num_n);
-        splits = g1;
-        est = est1;
-        if (pair_slots > 0 && best2 != ~0ull) {
-            const int g2 = static_cast<int>(best2 & 0xFFFFFull);
-            const float per2 = static_cast<float>((num_n + g2 - 1) / g2);
-            const float est2 = fmaxf(kPairTileCost * static_cast<float>(best2 >> 20),
-                                     hbm_tiles * per2 * g2 / num_n);
-            if (est2 < est1) {
-                mode = 2;
-                splits = g2;
-                est = est2;
-            }
-        }
-    }
-    __syncthreads();  // the shared keys may be reused by the next call
-    return est;  // estimated pass time in single-tile units (valid in thread 0)
-}
-
 __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p) {
     __shared__ int warp_sum[32];
-    __shared__ unsigned long long best_split;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int block_lo[kMaxBatch];  // RPD-block: first position of each canvas's active block
     pdl_trigger();  // successors may launch now; they wait for this grid before reading
@@ -184,68 +118,6 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
     }
 }
 
-// Lazy projection, second pass: compact the positions whose final-layer confidence lies in
-// their canvas's stability band (theta_c <= c < tau; Eq. 5 consults S_i only there) and set
-// the pass up over their K-1 earlier window layers.
-__global__ void __launch_bounds__(kCompactThreads, 1) k_band(BandParams p) {
-    __shared__ int warp_sum[32];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    pdl_trigger();  // successors may launch now; they wait for this grid before reading
-    pdl_wait();
-    const int nmt = p.meta[kMetaMasked];
-    const bool lazy_on = p.meta[kMetaLazy] != 0;  // else the first pass covered every layer
-    const float *final_p = p.row_pmax + static_cast<size_t>(p.K - 1) * nmt;
-    int carry = 0;
-    for (int base = 0; lazy_on && base < nmt; base += kCompactThreads * kCompactItems) {
-        const int q0 = base + tid * kCompactItems;
-        int f[kCompactItems];
-        int cnt = 0;
-#pragma unroll
-        for (int j = 0; j < kCompactItems; ++j) {
-            const int q = q0 + j;
-            f[j] = 0;
-            if (lazy_on && q < nmt && p.K > 1) {
-                const float c = final_p[q];
-                const int b = p.pos_of_q[q] / p.N;
-                f[j] = (c >= p.theta_c && c < p.tau[b]) ? 1 : 0;
-            }
-            cnt += f[j];
-        }
-        const int incl = warp_inclusive_scan(cnt, lane);
-        if (lane == 31) warp_sum[warp] = incl;
-        __syncthreads();
-        if (warp == 0) {
-            const int v = warp_sum[lane];
-            const int vi = warp_inclusive_scan(v, lane);
-            warp_sum[lane] = vi - v;
-        }
-        __syncthreads();
-        int excl = carry + warp_sum[warp] + incl - cnt;
-#pragma unroll
-        for (int j = 0; j < kCompactItems; ++j) {
-            if (f[j]) p.sel_q[excl] = q0 + j;
-            excl += f[j];
-        }
-        __syncthreads();
-        if (tid == kCompactThreads - 1) warp_sum[0] = excl;
-        __syncthreads();
-        carry = warp_sum[0];
-        __syncthreads();
-    }
-    const long long rows = static_cast<long long>(p.K - 1) * carry;
-    int mode, splits;
-    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.single_slots, p.pair_slots,
-                       p.hbm_tiles, mode, splits);
-    if (tid == 0) {
-        p.meta[kMetaRows] = static_cast<int>(rows);
-        p.meta[kMetaSplits] = splits;
-        p.meta[kMetaHeadMode] = mode;
-        p.meta[kMetaSel] = carry;
-        p.meta[kMetaLayer0] = 0;
-        p.meta[kMetaRowsTotal] += static_cast<int>(rows);
-    }
-}
-
 // One warp per row; the gain is staged once per CTA in shared memory and each lane keeps up
 // to kVecPerLane 16-byte loads of its row in flight before using any of them.
 constexpr int kNormThreads = 256;
@@ -313,10 +185,6 @@ __global__ void __launch_bounds__(kNormThreads) k_gather_norm(NormParams p) {
 
 cudaError_t launch_compact(const CompactParams &p, cudaStream_t s) {
     return launch_pdl(k_compact, dim3(1), dim3(kCompactThreads), 0, s, p);
-}
-
-cudaError_t launch_band(const BandParams &p, cudaStream_t s) {
-    return launch_pdl(k_band, dim3(1), dim3(kCompactThreads), 0, s, p);
 }
 
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s) {

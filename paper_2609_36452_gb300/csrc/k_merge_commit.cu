@@ -1,12 +1,12 @@
-// k_merge_commit.cu - cross-split merge of the online softmax statistics, then the
-// scoring, candidate flags, entropy prefix scan and commitment of §3.
+// k_merge_commit.cu - merge of the per-split softmax statistics, the lazy projection's band
+// selection, and the scoring, candidate flags, entropy prefix scan and commitment of §3.
 //
-// k_merge (one warp per projected row): combines the row's G partials (m, s, t, a) in
-//   log2 units into the row's argmax a, its probability 1/s and the entropy
-//   H = ln s - ln2 * t / s  (Eq. 1; p_v = 2^(x_v - m) / s).
-//   Merge rule for partials j: m = max m_j, alpha_j = 2^(m_j - m),
-//   s = sum alpha_j s_j, t = sum alpha_j (t_j + (m_j - m) s_j); argmax = lowest index among
-//   the partials attaining m.
+// k_merge (grid): combines each row's split partials of a projection pass into the row's
+//   argmax, its probability and its entropy (merge rule in step_common.cuh).
+//
+// k_band (one CTA; lazy projection only): selects the positions whose final confidence lies
+//   in their canvas's stability band theta_c <= c < tau (Eq. 5 reads S_i only there) and sets
+//   up the second pass over their earlier window layers.
 //
 // k_score_commit (one CTA per canvas, positions in blocked order across threads):
 //   y_i = argmax of the final layer, c_i its probability, H_i its entropy;
@@ -22,69 +22,94 @@
 //   later candidate sees at least that much entropy.
 //   If nothing is accepted and something is masked, commit the most confident of the
 //   first W masked positions (leftmost on ties, §3.2).  Then write the outputs, clear the
-//   committed mask bits and the per-canvas counters.
+//   committed mask bits and the per-canvas counters.  RPD-block skips the budget and takes
+//   the fallback over the active block.
 #include "ptx.cuh"
 #include "rpd_internal.h"
+#include "step_common.cuh"
 
 namespace rpd {
 namespace {
 
-constexpr float kLn2 = 0.6931471805599453f;
-
-struct Stat {
-    float m, s, t;
-    int a;
-};
-
-__device__ __forceinline__ Stat merge2(const Stat &x, const Stat &y) {
-    if (y.s <= 0.f) return x;
-    if (x.s <= 0.f) return y;
-    Stat r;
-    r.m = fmaxf(x.m, y.m);
-    const float dx = x.m - r.m, dy = y.m - r.m;
-    const float ax = exp2f(dx), ay = exp2f(dy);
-    r.s = ax * x.s + ay * y.s;
-    r.t = ax * fmaf(dx, x.s, x.t) + ay * fmaf(dy, y.s, y.t);
-    r.a = (x.m > y.m) ? x.a : (y.m > x.m) ? y.a : min(x.a, y.a);
-    return r;
-}
-
-__global__ void __launch_bounds__(256) k_merge(MergeParams p) {
+// Grid-wide merge of the current projection pass (every row of every canvas).
+__global__ void __launch_bounds__(256) k_merge(MergeArgs mg, const int32_t *meta,
+                                               const int32_t *sel_list) {
     pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
-    const int rows = p.meta[kMetaRows];
-    const int splits = p.meta[kMetaSplits];
+    merge_pass_rows(mg, meta, sel_list, 0, meta[kMetaSel], blockIdx.x, gridDim.x);
+}
+
+constexpr int kBandThreads = 1024;
+constexpr int kBandItems = 4;
+
+__global__ void __launch_bounds__(kBandThreads, 1) k_band(BandParams p) {
+    __shared__ int warp_sum[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
+    pdl_wait();
     const int nmt = p.meta[kMetaMasked];
-    const int sel = p.meta[kMetaSel];
-    const int layer0 = p.meta[kMetaLayer0];
-    const int lane = threadIdx.x & 31;
-    const int wpc = blockDim.x >> 5;
-    for (int r = blockIdx.x * wpc + (threadIdx.x >> 5); r < rows; r += gridDim.x * wpc) {
-        // this pass's row r is layer layer0 + r / sel of compact position sel_list[r % sel]
-        const int kr = r / sel;
-        const int sr = r - kr * sel;
-        const size_t out = static_cast<size_t>(layer0 + kr) * nmt + (p.sel_list ? p.sel_list[sr] : sr);
-        Stat acc{-INFINITY, 0.f, 0.f, 0x7fffffff};
-        const float4 *row = p.partials + static_cast<size_t>(r) * p.max_splits;
-        for (int g = lane; g < splits; g += 32) {
-            const float4 v = row[g];
-            acc = merge2(acc, Stat{v.x, v.y, v.z, __float_as_int(v.w)});
-        }
+    const bool lazy_on = p.meta[kMetaLazy] != 0;  // else the first pass covered every layer
+    // 1. band positions, in compact order (the first pass was merged by k_merge)
+    const float *final_p = p.mg.row_pmax + static_cast<size_t>(p.K - 1) * nmt;
+    int carry = 0;
+    for (int base = 0; lazy_on && base < nmt; base += kBandThreads * kBandItems) {
+        const int q0 = base + tid * kBandItems;
+        int f[kBandItems];
+        int cnt = 0;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            Stat other;
-            other.m = __shfl_xor_sync(0xffffffffu, acc.m, o);
-            other.s = __shfl_xor_sync(0xffffffffu, acc.s, o);
-            other.t = __shfl_xor_sync(0xffffffffu, acc.t, o);
-            other.a = __shfl_xor_sync(0xffffffffu, acc.a, o);
-            // combine in lane order so every lane ends with the same bits
-            acc = (lane & o) ? merge2(other, acc) : merge2(acc, other);
+        for (int j = 0; j < kBandItems; ++j) {
+            const int q = q0 + j;
+            f[j] = 0;
+            if (q < nmt && p.K > 1) {
+                const float c = final_p[q];
+                const int b = p.pos_of_q[q] / p.N;
+                f[j] = (c >= p.theta_c && c < p.tau[b]) ? 1 : 0;
+            }
+            cnt += f[j];
         }
-        if (lane == 0) {
-            p.row_arg[out] = acc.a;
-            p.row_pmax[out] = 1.0f / acc.s;
-            p.row_H[out] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
+        const int incl = warp_inclusive_scan(cnt, lane);
+        if (lane == 31) warp_sum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            const int v = warp_sum[lane];
+            const int vi = warp_inclusive_scan(v, lane);
+            warp_sum[lane] = vi - v;
         }
+        __syncthreads();
+        int excl = carry + warp_sum[warp] + incl - cnt;
+#pragma unroll
+        for (int j = 0; j < kBandItems; ++j) {
+            if (f[j]) p.sel_q[excl] = q0 + j;
+            excl += f[j];
+        }
+        __syncthreads();
+        if (tid == kBandThreads - 1) warp_sum[0] = excl;
+        __syncthreads();
+        carry = warp_sum[0];
+        __syncthreads();
+    }
+    // 2. each canvas's range in the band list (the list is sorted, canvases are contiguous)
+    for (int b = tid; b <= p.B; b += kBandThreads) {
+        const int key = p.canvas_off[b];
+        int lo = 0, hi = carry;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (p.sel_q[mid] < key) lo = mid + 1; else hi = mid;
+        }
+        p.band_off[b] = lo;
+    }
+    // 3. the second pass: the K-1 earlier window layers of the band positions
+    const long long rows = static_cast<long long>(p.K - 1) * carry;
+    int mode, splits;
+    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.single_slots, p.pair_slots,
+                       p.hbm_tiles, mode, splits);
+    if (tid == 0) {
+        p.meta[kMetaRows] = static_cast<int>(rows);
+        p.meta[kMetaSplits] = splits;
+        p.meta[kMetaHeadMode] = mode;
+        p.meta[kMetaSel] = carry;
+        p.meta[kMetaLayer0] = 0;
+        p.meta[kMetaRowsTotal] += static_cast<int>(rows);
     }
 }
 
@@ -361,8 +386,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
 
 }  // namespace
 
-cudaError_t launch_merge(const MergeParams &p, int grid, cudaStream_t s) {
-    return launch_pdl(k_merge, dim3(grid), dim3(256), 0, s, p);
+cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,
+                         int grid, cudaStream_t s) {
+    return launch_pdl(k_merge, dim3(grid), dim3(256), 0, s, mg, meta, sel_list);
+}
+
+cudaError_t launch_band(const BandParams &p, cudaStream_t s) {
+    return launch_pdl(k_band, dim3(1), dim3(kBandThreads), 0, s, p);
 }
 
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s) {

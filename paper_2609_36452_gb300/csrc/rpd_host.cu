@@ -96,6 +96,7 @@ struct rpd_ctx {
     float *row_pmax = nullptr, *row_H = nullptr;
     int32_t *q_of_pos = nullptr, *pos_of_q = nullptr, *canvas_off = nullptr, *meta = nullptr;
     int32_t *sel_q = nullptr;  // lazy projection: compact indices of the band positions
+    int32_t *band_off = nullptr;  // lazy projection: [B+1] each canvas's first band entry
     int projection = RPD_PROJECT_ALL;
     CUtensorMap tmU{}, tmW{}, tmW_pair{};
     int pair_grid = 0;   // CTAs of the CTA-pair head kernel (2 x resident pairs; 0 = none)
@@ -112,7 +113,7 @@ struct rpd_ctx {
 
     void free_scratch() {
         void *ptrs[] = {u, inv_rms, partials, row_arg, row_pmax, row_H, q_of_pos, pos_of_q,
-                        canvas_off, meta, sel_q};
+                        canvas_off, meta, sel_q, band_off};
         for (void *p : ptrs)
             if (p) cudaFree(p);
         u = nullptr;
@@ -120,7 +121,7 @@ struct rpd_ctx {
         partials = nullptr;
         row_arg = nullptr;
         row_pmax = row_H = nullptr;
-        q_of_pos = pos_of_q = canvas_off = meta = sel_q = nullptr;
+        q_of_pos = pos_of_q = canvas_off = meta = sel_q = band_off = nullptr;
         cap_bn = cap_b = cap_rows = 0;
     }
 };
@@ -155,6 +156,7 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
         {reinterpret_cast<void **>(&c->pos_of_q), static_cast<size_t>(new_bn) * 4},
         {reinterpret_cast<void **>(&c->sel_q), static_cast<size_t>(new_bn) * 4},
         {reinterpret_cast<void **>(&c->canvas_off), static_cast<size_t>(new_b + 1) * 4},
+        {reinterpret_cast<void **>(&c->band_off), static_cast<size_t>(new_b + 1) * 4},
         {reinterpret_cast<void **>(&c->meta), kMetaWords * 4},
     };
     for (auto &a : allocs) {
@@ -264,8 +266,9 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         e = launch_compact(cp, c->stream);
     }
     if (e != cudaSuccess) return cuda_fail(e, "compaction launch");
-    // One projection pass: gather + RMSNorm prologue, head statistics, merge.  Rows, layers and
-    // positions of the pass come from the device-side meta words.
+    // One projection pass: gather + RMSNorm prologue, head statistics, merge.  Rows, layers
+    // and positions of the pass come from the device-side meta words.
+    const MergeArgs mg{c->partials, c->max_splits, c->row_arg, c->row_pmax, c->row_H};
     auto pass = [&](const int32_t *sel_list) -> cudaError_t {
         cudaError_t err;
         {
@@ -287,9 +290,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         }
         if (err != cudaSuccess) return err;
         KernelTimer t(c, 2);
-        MergeParams mp{c->partials, sel_list, c->meta, c->row_arg, c->row_pmax, c->row_H,
-                       c->max_splits};
-        return launch_merge(mp, c->num_sms * 8, c->stream);
+        return launch_merge(mg, c->meta, sel_list, c->num_sms * 4, c->stream);
     };
     e = pass(nullptr);
     if (e == cudaSuccess && lazy) {
@@ -297,9 +298,12 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             KernelTimer t(c, 2);
             BandParams bp{};
             bp.meta = c->meta;
+            bp.mg = mg;
             bp.pos_of_q = c->pos_of_q;
-            bp.row_pmax = c->row_pmax;
+            bp.canvas_off = c->canvas_off;
             bp.sel_q = c->sel_q;
+            bp.band_off = c->band_off;
+            bp.B = B;
             bp.N = N;
             bp.K = c->K;
             bp.theta_c = c->rule.theta_c;

@@ -70,12 +70,24 @@ constexpr float kLazyBandGuess = 0.25f;
 // Second pass of lazy projection: selects the positions whose final confidence lies in the
 // stability band theta_c <= c < tau of their canvas and sets up the pass over their earlier
 // window layers (tiling, split count, row mapping).
+// Where merged per-row statistics go: split partials (log2 units) in, argmax / max
+// probability / entropy per (layer, compact position) out, at layer * NMT + q.
+struct MergeArgs {
+    const float4 *partials;  // [rows][max_splits]
+    int max_splits;
+    int32_t *row_arg;
+    float *row_pmax;
+    float *row_H;
+};
+
 struct BandParams {
     int32_t *meta;
+    MergeArgs mg;              // merged first-pass statistics (final-layer confidences)
     const int32_t *pos_of_q;   // [NMT] flat position b*N+i of compact index q
-    const float *row_pmax;     // final-layer probabilities at (K-1)*NMT + q
+    const int32_t *canvas_off; // [B+1] first compact index of each canvas
     int32_t *sel_q;            // out: compact indices of the band positions
-    int N, K;
+    int32_t *band_off;         // out: [B+1] first band entry of each canvas
+    int B, N, K;
     float theta_c;
     int num_n_tiles, max_splits, single_slots, pair_slots;
     float hbm_tiles;
@@ -92,7 +104,7 @@ constexpr double kHeadStreamBytesPerSec = 6.5e12;
 
 // Row r of a projection pass: layer k = meta[kMetaLayer0] + r / S and position
 // q = sel[r % S] (sel = the pass's list of compact indices, or the identity when null),
-// S = meta[kMetaSel]; its statistics land at k * NMT + q.
+// S = meta[kMetaSel]; its merged statistics land at k * NMT + q.
 struct NormParams {
     const __nv_bfloat16 *hidden;  // [K][B*N][d]
     const __nv_bfloat16 *gain;    // [d]
@@ -119,16 +131,6 @@ inline float head_stream_in_tiles(int V, int d, int num_sms) {
     const double t_tile = 2.0 * kTileM * kTileN * static_cast<double>(d) / kSingleTileFlopsPerSm;
     return static_cast<float>(t_hbm / t_tile);
 }
-
-struct MergeParams {
-    const float4 *partials;
-    const int32_t *sel_list;  // as in NormParams
-    const int32_t *meta;
-    int32_t *row_arg;   // [rows]
-    float *row_pmax;    // [rows]
-    float *row_H;       // [rows]
-    int max_splits;
-};
 
 struct ScoreParams {
     uint8_t *mask;              // [B][N] in/out
@@ -182,7 +184,8 @@ cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tm
                                    const HeadParams &p, int grid, cudaStream_t s);
 // Largest number of CTA pairs of the pair kernel that can be resident at once.
 int head_stats_pair_max_clusters();
-cudaError_t launch_merge(const MergeParams &p, int grid, cudaStream_t s);
+cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,
+                         int grid, cudaStream_t s);
 cudaError_t launch_band(const BandParams &p, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
 

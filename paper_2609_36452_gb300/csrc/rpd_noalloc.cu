@@ -217,10 +217,9 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         if (e == cudaSuccess && pair_slots > 0)
             e = launch_head_stats_pair(tmU, tmW_pair, hp, dev->pair_grid, stream);
     }
-    if (e == cudaSuccess) {
-        MergeParams mp{partials, nullptr, meta, row_arg, row_pmax, row_H, splits};
-        e = launch_merge(mp, dev->num_sms * 8, stream);
-    }
+    if (e == cudaSuccess)
+        e = launch_merge(MergeArgs{partials, splits, row_arg, row_pmax, row_H}, meta, nullptr,
+                         dev->num_sms * 4, stream);
     if (e == cudaSuccess) {
         ScoreParams sp{};
         sp.mask = mask;
