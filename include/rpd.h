@@ -155,7 +155,9 @@ int rpd_step(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau, 
 /* B independent canvases of N positions in one step; the head is read once for all.
  *   hidden [K][B][N][d] bf16 device; mask, out_commit, out_token [B][N] device;
  *   tau, budget [B] HOST arrays (per-canvas theta_h and beta); out_stats [B] device.
- * Requires 1 <= B <= 128. */
+ * Requires 1 <= B <= 128.  Canvases of different lengths are padded to a common N with mask
+ * 0: unmasked positions are never projected, scored, counted in E_i or committed, so each
+ * canvas's result is that of its unpadded length. */
 int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int N,
                      const float *tau, const float *budget, uint8_t *out_commit,
                      int32_t *out_token, rpd_stats *out_stats);

@@ -420,3 +420,34 @@ def test_auto_projection_picks_per_step(llada_head):
             assert b["stats"]["n_rows"] < case["K"] * nm
         else:
             assert b["stats"]["n_rows"] == case["K"] * nm
+
+
+def test_batched_heterogeneous_lengths():
+    """Canvases of different lengths in one batched step: each is padded to N with mask 0
+    (padding is never projected, scored, counted in the budget or committed) and must equal
+    the oracle on the unpadded canvas."""
+    K, N, d, V = 3, 100, 256, 2048
+    lengths = [100, 64, 37]
+    B = len(lengths)
+    W, g = WL.make_head(V, d, 93, w_std=0.08)
+    hidden = torch.empty(K, B, N, d, dtype=torch.bfloat16)
+    masks = torch.zeros(B, N, dtype=torch.uint8)
+    for b, nb in enumerate(lengths):
+        cv = WL.make_hidden(W, K, N, 900 + b, WL.u_profile(N, 0.5, 3.0),
+                            WL.calibrated_sigma(V, d, 0.08, 3.0), flip_frac=0.1)
+        hidden[:, b] = cv.hidden
+        hidden[:, b, nb:] = 0          # padding rows carry nothing
+        masks[b, :nb] = WL.uniform_fraction_mask(nb, 0.8, 950 + b)
+    taus, budgets = [0.9, 0.85, 0.9], [1.0, 2.0, 0.5]
+    runner = GpuRunner(W, g, K)
+    try:
+        outs = runner.step_batched(hidden, masks, taus, budgets)
+    finally:
+        runner.close()
+    for b, nb in enumerate(lengths):
+        ref = O.rpd_step(bits(hidden[:, b, :nb]), masks[b, :nb].numpy(), bits(g), bits(W), 1e-6,
+                         taus[b], budgets[b], "llada")
+        got = {k: (v[:nb] if isinstance(v, np.ndarray) and v.ndim == 1 else
+                   (v[:, :nb] if isinstance(v, np.ndarray) else v)) for k, v in outs[b].items()}
+        compare_step(ref, got)
+        assert np.all(outs[b]["commit"][nb:] == 0) and np.all(outs[b]["new_mask"][nb:] == 0)
