@@ -133,6 +133,16 @@ int rpd_reserve(rpd_ctx *ctx, int B, int N);
 #define RPD_PROJECT_AUTO 2
 int rpd_set_projection(rpd_ctx *ctx, int mode);
 
+/* Diagnostics.  Every wait inside the step's kernels (mbarrier waits of the head kernels) is
+ * bounded; when one runs out the kernel stops, drains what it has in flight, frees its
+ * tensor memory and latches RPD_ERR_TIMEOUT in rpd_stats.status (the other outputs of that
+ * step are then meaningless); the context stays usable.
+ *   rpd_set_wait_limit: the bound, in microseconds (default 2 000 000), >= 1000.
+ *   rpd_inject_stall:  the next step's head kernels issue no loads at all, so their waits run
+ *                      out and the step reports RPD_ERR_TIMEOUT; used to test the path. */
+int rpd_set_wait_limit(rpd_ctx *ctx, int64_t microseconds);
+int rpd_inject_stall(rpd_ctx *ctx);
+
 /* Install (or with NULL, clear) the optional per-position outputs. */
 int rpd_set_debug(rpd_ctx *ctx, const rpd_debug *debug);
 

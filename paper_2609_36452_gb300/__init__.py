@@ -15,7 +15,7 @@ __all__ = [
     "RPD_OK", "RPD_ERR_INVALID_ARGUMENT", "RPD_ERR_NO_HEAD", "RPD_ERR_CUDA",
     "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
-    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_step",
+    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_profile_enable", "rpd_kernel_times",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
@@ -89,6 +89,8 @@ def _load():
         "rpd_reserve": (i32, [vp, i32, i32]),
         "rpd_set_debug": (i32, [vp, ctypes.POINTER(RpdDebug)]),
         "rpd_set_projection": (i32, [vp, i32]),
+        "rpd_set_wait_limit": (i32, [vp, ctypes.c_int64]),
+        "rpd_inject_stall": (i32, [vp]),
         "rpd_step": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_step_batched": (i32, [vp, vp, vp, i32, i32, vp, vp, vp, vp, vp]),
         "rpd_step_host": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
@@ -118,6 +120,8 @@ rpd_set_stream = lib.rpd_set_stream
 rpd_reserve = lib.rpd_reserve
 rpd_set_debug = lib.rpd_set_debug
 rpd_set_projection = lib.rpd_set_projection
+rpd_set_wait_limit = lib.rpd_set_wait_limit
+rpd_inject_stall = lib.rpd_inject_stall
 rpd_step = lib.rpd_step
 rpd_step_batched = lib.rpd_step_batched
 rpd_step_host = lib.rpd_step_host
@@ -190,6 +194,14 @@ class Rpd:
         if isinstance(mode, bool):
             mode = "lazy" if mode else "all"
         _check(rpd_set_projection(self.handle, PROJECTION_MODES[mode]))
+
+    def set_wait_limit(self, microseconds: int):
+        _check(rpd_set_wait_limit(self.handle, int(microseconds)))
+
+    def inject_stall(self):
+        """Diagnostics: the next step's head kernels issue no loads; the step reports
+        RPD_ERR_TIMEOUT once its bounded waits run out."""
+        _check(rpd_inject_stall(self.handle))
 
     def reserve(self, B: int, N: int):
         _check(rpd_reserve(self.handle, B, N))

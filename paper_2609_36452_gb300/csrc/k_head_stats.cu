@@ -130,7 +130,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (warp == 0) {
-        if (lane == 0) {
+        if (lane == 0 && !p.stall) {
             // ---------------------------------------------------------------- TMA producer
             int stage = 0;
             uint32_t phase = 0;
@@ -141,7 +141,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 tw.unit(u, m, n0, n1);
                 for (int n = n0; ok && n < n1; ++n) {
                     for (int kb = 0; kb < num_kb; ++kb) {
-                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
+                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit_ns)) {
                             ok = false;
                             break;
                         }
@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             // normal path they all have, since the MMA consumed them).
             for (int s = 0; s < kStages; ++s) {
                 const long long n_s = fills / kStages + (s < fills % kStages ? 1 : 0);
-                if (n_s > 0) mbar_wait_drain(&full[s], static_cast<uint32_t>((n_s - 1) & 1), kWaitLimitNs);
+                if (n_s > 0) mbar_wait_drain(&full[s], static_cast<uint32_t>((n_s - 1) & 1), p.wait_limit_ns);
             }
         }
     } else if (warp == 1) {
@@ -180,14 +180,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                     const uint32_t acc = tile_iter & 1u;
                     const uint32_t acc_phase = (tile_iter >> 1) & 1u;
                     if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
-                                           kWaitLimitNs)) {
+                                           p.wait_limit_ns)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after_sync();
                     const uint32_t d_tmem = tmem_base + acc * kTileN;
                     for (int kb = 0; kb < num_kb; ++kb) {
-                        if (!mbar_wait_bounded(&full[stage], phase, abort_flag, kWaitLimitNs)) {
+                        if (!mbar_wait_bounded(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
                             ok = false;
                             break;
                         }
@@ -212,7 +212,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             }
             // Drain: wait until every MMA this thread issued has completed.
             umma_commit(drain);
-            mbar_wait_drain(drain, 0, kWaitLimitNs);
+            mbar_wait_drain(drain, 0, p.wait_limit_ns);
         }
     } else {
         // -------------------------------------------------------------------- epilogue
@@ -232,7 +232,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             for (int n = n0; n < n1; ++n, ++tile_iter) {
                 const uint32_t acc = tile_iter & 1u;
                 const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, kWaitLimitNs)) {
+                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
                     ok = false;
                     break;
                 }
@@ -343,7 +343,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (warp == 0) {
-        if (lane == 0) {
+        if (lane == 0 && !p.stall) {
             // ------------------------------------------------------- TMA producer (both CTAs)
             const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);
             int stage = 0;
@@ -355,7 +355,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 tw.unit(u, m, n0, n1);
                 for (int n = n0; ok && n < n1; ++n) {
                     for (int kb = 0; kb < num_kb; ++kb) {
-                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
+                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit_ns)) {
                             ok = false;
                             break;
                         }
@@ -379,7 +379,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             for (int s = 0; s < kPairStages; ++s) {
                 const long long n_s = fills / kPairStages + (s < fills % kPairStages ? 1 : 0);
                 if (n_s > 0)
-                    mbar_wait_drain(&empty[s], static_cast<uint32_t>((n_s - 1) & 1), kWaitLimitNs / 8);
+                    mbar_wait_drain(&empty[s], static_cast<uint32_t>((n_s - 1) & 1), p.wait_limit_ns / 8);
             }
         }
     } else if (warp == 1) {
@@ -398,14 +398,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                         const uint32_t acc = tile_iter & 1u;
                         const uint32_t acc_phase = (tile_iter >> 1) & 1u;
                         if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
-                                               kWaitLimitNs)) {
+                                               p.wait_limit_ns)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after_sync();
                         const uint32_t d_tmem = tmem_base + acc * kTileN;
                         for (int kb = 0; kb < num_kb; ++kb) {
-                            if (!mbar_wait_bounded(&full[stage], phase, abort_flag, kWaitLimitNs)) {
+                            if (!mbar_wait_bounded(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
                                 ok = false;
                                 break;
                             }
@@ -431,7 +431,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 umma_commit_pair_multicast(drain, 0x3);
             }
             // Both CTAs: every MMA writing this CTA's TMEM has completed before it is freed.
-            mbar_wait_drain(drain, 0, kWaitLimitNs);
+            mbar_wait_drain(drain, 0, p.wait_limit_ns);
         }
     } else {
         // ---------------------------------------------------------- epilogue (both CTAs)
@@ -452,7 +452,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             for (int n = n0; n < n1; ++n, ++tile_iter) {
                 const uint32_t acc = tile_iter & 1u;
                 const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, kWaitLimitNs)) {
+                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
                     ok = false;
                     break;
                 }

@@ -98,6 +98,8 @@ struct rpd_ctx {
     int32_t *sel_q = nullptr;  // lazy projection: compact indices of the band positions
     int32_t *band_off = nullptr;  // lazy projection: [B+1] each canvas's first band entry
     int projection = RPD_PROJECT_ALL;
+    uint64_t wait_limit_ns = kWaitLimitNs;
+    bool stall_next = false;  // diagnostics: the next step's head kernels issue no loads
     CUtensorMap tmU{}, tmW{}, tmW_pair{};
     int pair_grid = 0;   // CTAs of the CTA-pair head kernel (2 x resident pairs; 0 = none)
 
@@ -281,7 +283,8 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         if (err != cudaSuccess) return err;
         {
             KernelTimer t(c, 1);
-            HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits};
+            HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits,
+                          c->wait_limit_ns, c->stall_next ? 1 : 0};
             // Both tilings are launched; each reads the choice made on the device for this
             // pass's row count and the other returns at once.
             err = launch_head_stats(c->tmU, c->tmW, hp, c->num_sms, c->stream);
@@ -317,6 +320,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         }
         if (e == cudaSuccess) e = pass(c->sel_q);
     }
+    c->stall_next = false;
     if (e != cudaSuccess) return cuda_fail(e, "projection launch");
     {
         KernelTimer t(c, 3);
@@ -453,6 +457,19 @@ int rpd_set_projection(rpd_ctx *c, int mode) {
     if (mode != RPD_PROJECT_ALL && mode != RPD_PROJECT_LAZY && mode != RPD_PROJECT_AUTO)
         return fail(RPD_ERR_INVALID_ARGUMENT, "unknown projection mode %d", mode);
     c->projection = mode;
+    return RPD_OK;
+}
+
+int rpd_set_wait_limit(rpd_ctx *c, int64_t microseconds) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (microseconds < 1000) return fail(RPD_ERR_INVALID_ARGUMENT, "wait limit must be >= 1000 us");
+    c->wait_limit_ns = static_cast<uint64_t>(microseconds) * 1000ull;
+    return RPD_OK;
+}
+
+int rpd_inject_stall(rpd_ctx *c) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    c->stall_next = true;
     return RPD_OK;
 }
 

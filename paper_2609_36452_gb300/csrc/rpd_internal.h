@@ -122,6 +122,8 @@ struct HeadParams {
     float4 *partials;      // [rows][max_splits]: (max, sum, tsum, argmax bits), log2 units
     int32_t *meta;
     int V, d, max_splits;
+    uint64_t wait_limit_ns;  // bound on every mbarrier wait
+    int stall;               // diagnostics: issue no loads (the waits run out)
 };
 
 // Time to stream the head once, in units of one single-CTA tile's MMA time.

@@ -212,7 +212,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         e = launch_gather_norm(np, dev->num_sms * 8, stream);
     }
     if (e == cudaSuccess) {
-        HeadParams hp{inv_rms, partials, meta, V, d, splits};
+        HeadParams hp{inv_rms, partials, meta, V, d, splits, kWaitLimitNs, 0};
         e = launch_head_stats(tmU, tmW, hp, dev->num_sms, stream);
         if (e == cudaSuccess && pair_slots > 0)
             e = launch_head_stats_pair(tmU, tmW_pair, hp, dev->pair_grid, stream);

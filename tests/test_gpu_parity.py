@@ -451,3 +451,47 @@ def test_batched_heterogeneous_lengths():
                    (v[:, :nb] if isinstance(v, np.ndarray) else v)) for k, v in outs[b].items()}
         compare_step(ref, got)
         assert np.all(outs[b]["commit"][nb:] == 0) and np.all(outs[b]["new_mask"][nb:] == 0)
+
+
+# ----------------------------------------------------------------------------- failure detection
+
+@pytest.mark.parametrize("N,K", [(256, 4), (32, 2)])   # CTA-pair and single-CTA head tilings
+def test_stalled_head_reports_timeout_and_context_recovers(N, K):
+    """A step whose head kernels issue no loads: their bounded waits run out, the step reports
+    RPD_ERR_TIMEOUT in rpd_stats.status without faulting or hanging, and the next step on the
+    same context is correct again."""
+    import paper_2609_36452_gb300 as rpd
+    case = small_case(301 + N, K=K, N=N)
+    runner = GpuRunner(case["W"], case["g"], K)
+    try:
+        runner.ctx.set_wait_limit(20000)          # 20 ms
+        runner.ctx.inject_stall()
+        bad = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
+        assert bad["stats"]["status"] == rpd.RPD_ERR_TIMEOUT
+        good = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
+    finally:
+        runner.close()
+    assert good["stats"]["status"] == 0
+    compare_step(oracle_step(case), good)
+
+
+def test_exact_argmax_tie_takes_lowest_token():
+    """Two identical head rows give bitwise-equal logits; the argmax is the lower token index,
+    on every layer, as the oracle's reading (first occurrence) requires."""
+    K, N, d, V = 2, 8, 128, 2048
+    W, g = WL.make_head(V, d, 99, w_std=0.08)
+    lo, hi = 100, 1900          # different vocabulary tiles and splits
+    W[hi] = W[lo]
+    targets = torch.full((N,), lo, dtype=torch.long)
+    cv = WL.make_hidden(W, K, N, 98, torch.full((N,), 3.0), WL.calibrated_sigma(V, d, 0.08, 3.0),
+                        targets=targets)
+    mask = torch.ones(N, dtype=torch.uint8)
+    runner = GpuRunner(W, g, K)
+    try:
+        got = runner.step(cv.hidden, mask, 0.9, 1.0)
+    finally:
+        runner.close()
+    ref = O.rpd_step(bits(cv.hidden), mask.numpy(), bits(g), bits(W), 1e-6, 0.9, 1.0, "llada")
+    assert np.all(ref.layer_argmax == lo) and np.all(ref.layer_gap == 0.0)
+    assert np.all(got["layer_argmax"] == lo)
+    assert np.all(got["token"][got["commit"] == 1] == lo)
