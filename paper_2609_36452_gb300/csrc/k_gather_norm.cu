@@ -129,13 +129,14 @@ __global__ void __launch_bounds__(kNormThreads) k_gather_norm(NormParams p) {
     const int warps_per_cta = blockDim.x >> 5;
     const int nvec = p.d >> 3;  // 8 bf16 per 16-byte vector
     const uint4 *__restrict__ gvec = reinterpret_cast<const uint4 *>(p.gain);
-    for (int v = threadIdx.x; v < nvec; v += blockDim.x) g_smem[v] = __ldg(gvec + v);
     pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
+    const int rows = p.meta[kMetaRows];
+    if (static_cast<long long>(blockIdx.x) * warps_per_cta >= rows) return;  // no row here
+    for (int v = threadIdx.x; v < nvec; v += blockDim.x) g_smem[v] = __ldg(gvec + v);
     __syncthreads();
     const int sel = p.meta[kMetaSel];
     const int layer0 = p.meta[kMetaLayer0];
-    const int rows = p.meta[kMetaRows];
     for (int r = blockIdx.x * warps_per_cta + (threadIdx.x >> 5); r < rows;
          r += gridDim.x * warps_per_cta) {
         const int kr = r / sel;

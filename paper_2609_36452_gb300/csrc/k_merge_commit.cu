@@ -182,8 +182,10 @@ __device__ __forceinline__ int4 block_sum4(int4 v, int4 *sh) {
 
 constexpr int kLayerBatch = 8;  // window layers whose statistics are loaded together
 
+// kMaxItems positions per thread at most (N <= kMaxItems * blockDim.x); instantiated for
+// 1, 2, 4 and 8 so that short canvases carry no unused per-item state.
+template <int kMaxItems>
 __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p) {
-    constexpr int kMaxItems = kMaxCanvas / kScoreThreads;
     __shared__ ScanPair sh_scan[33];
     __shared__ int4 sh_sum[32];
     __shared__ int first_reject;
@@ -216,11 +218,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
         const int i = i0 + j;
         if (j >= items || i >= N) continue;
         const size_t pos = static_cast<size_t>(b) * N + i;
+        // both loads issued together (q_of_pos is -1 wherever the mask is 0)
+        const int q_raw = p.q_of_pos[pos];
         const bool is_masked = mask[i] != 0;
         n_masked_all += is_masked;
         // Scored positions: every masked one, or (RPD-block) the active block's masked ones,
         // which are exactly those the compaction kept.
-        const int q = is_masked ? p.q_of_pos[pos] : -1;
+        const int q = is_masked ? q_raw : -1;
         masked[j] = q >= 0;
         int ki = 0;
         float r = 0.f, s = 0.f;
@@ -397,7 +401,11 @@ cudaError_t launch_band(const BandParams &p, cudaStream_t s) {
 
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s) {
     const int threads = p.N >= kScoreThreads ? kScoreThreads : ((p.N + 31) / 32) * 32;
-    return launch_pdl(k_score_commit, dim3(p.B), dim3(threads), 0, s, p);
+    const int items = (p.N + threads - 1) / threads;
+    if (items <= 1) return launch_pdl(k_score_commit<1>, dim3(p.B), dim3(threads), 0, s, p);
+    if (items <= 2) return launch_pdl(k_score_commit<2>, dim3(p.B), dim3(threads), 0, s, p);
+    if (items <= 4) return launch_pdl(k_score_commit<4>, dim3(p.B), dim3(threads), 0, s, p);
+    return launch_pdl(k_score_commit<kMaxCanvas / kScoreThreads>, dim3(p.B), dim3(threads), 0, s, p);
 }
 
 }  // namespace rpd

@@ -278,7 +278,10 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
                           static_cast<const __nv_bfloat16 *>(c->g), c->pos_of_q, sel_list, c->meta,
                           c->u, c->inv_rms, bn, c->d, c->eps};
-            err = launch_gather_norm(np, c->num_sms * 8, c->stream);
+            // one warp per row: no more CTAs than the largest possible row count needs
+            const long long max_rows = static_cast<long long>(c->K) * bn;
+            const int grid = static_cast<int>(std::min<long long>(c->num_sms * 8, (max_rows + 7) / 8));
+            err = launch_gather_norm(np, grid, c->stream);
         }
         if (err != cudaSuccess) return err;
         {

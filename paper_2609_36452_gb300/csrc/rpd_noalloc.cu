@@ -209,7 +209,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
                       static_cast<const __nv_bfloat16 *>(g_norm), pos_of_q, nullptr, meta, u,
                       inv_rms, N, d, eps};
-        e = launch_gather_norm(np, dev->num_sms * 8, stream);
+        e = launch_gather_norm(np, std::min(dev->num_sms * 8, (K * N + 7) / 8), stream);
     }
     if (e == cudaSuccess) {
         HeadParams hp{inv_rms, partials, meta, V, d, splits, kWaitLimitNs, 0};
