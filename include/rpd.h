@@ -172,9 +172,11 @@ int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int
                      const float *tau, const float *budget, uint8_t *out_commit,
                      int32_t *out_token, rpd_stats *out_stats);
 
-/* rpd_step with HOST buffers: copies hidden and mask in, runs the step, copies mask,
- * out_commit, out_token and out_stats back, and returns after the stream has finished.
- * Staging buffers are owned by the context (grown on demand).  mask is in/out. */
+/* rpd_step with HOST buffers: copies hidden, mask and out_token in, runs the step, copies
+ * mask, out_commit, out_token and out_stats back, and returns after the stream has finished.
+ * mask and out_token are in/out: out_token (the canvas) changes only at committed positions.
+ * Staging buffers are owned by the context (grown on demand; the first call of a larger size
+ * allocates). */
 int rpd_step_host(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau,
                   float budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats);
 

@@ -190,7 +190,7 @@ cudaError_t launch_compact(const CompactParams &p, cudaStream_t s) {
 
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s) {
     const size_t smem = static_cast<size_t>(p.d) * 2;  // the gain, staged once per CTA
-    if (smem > 48 * 1024) {
+    if (smem > 48 * 1024) {  // set on the current device before every such launch
         cudaError_t e = cudaFuncSetAttribute(k_gather_norm, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(smem));
         if (e != cudaSuccess) return e;

@@ -20,6 +20,8 @@
 // Two 256-column fp32 accumulators (512 TMEM columns) let the epilogue of one tile run
 // under the MMAs of the next.  Every wait is bounded; a timeout latches RPD_ERR_TIMEOUT
 // in the step's status word and the CTA drains and exits.
+#include <atomic>
+
 #include "ptx.cuh"
 #include "rpd_internal.h"
 
@@ -493,17 +495,35 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     }
 }
 
+// Per-device one-time settings (the dynamic shared-memory opt-in is a property of the
+// kernel on each device).
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_single_ready[kMaxDevices];
+std::atomic<int> g_pair_ready[kMaxDevices];
+std::atomic<int> g_pair_clusters[kMaxDevices];  // resident pairs + 1 (0: not queried yet)
+
+int current_device() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return -1;
+    return dev;
+}
+
+cudaError_t opt_in_smem(const void *kernel, int bytes, std::atomic<int> *ready) {
+    const int dev = current_device();
+    if (dev < 0) return cudaErrorInvalidDevice;
+    if (ready[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) ready[dev].store(1, std::memory_order_release);
+    return e;
+}
+
 }  // namespace
 
 cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, const HeadParams &p,
                               int grid, cudaStream_t s) {
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(k_head_stats, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kHeadSmemBytes);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(k_head_stats), kHeadSmemBytes,
+                                g_single_ready);
+    if (e != cudaSuccess) return e;
     return launch_pdl(k_head_stats, dim3(grid), dim3(kHeadThreads), kHeadSmemBytes, s, tmU, tmW, p);
 }
 
@@ -512,11 +532,13 @@ cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, co
 namespace rpd {
 
 int head_stats_pair_max_clusters() {
-    static int cached = -1;
-    if (cached >= 0) return cached;
-    cudaError_t e = cudaFuncSetAttribute(k_head_stats_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kPairSmemBytes);
-    if (e != cudaSuccess) return 0;
+    const int dev = current_device();
+    if (dev < 0) return 0;
+    const int cached = g_pair_clusters[dev].load(std::memory_order_acquire);
+    if (cached > 0) return cached - 1;
+    if (opt_in_smem(reinterpret_cast<const void *>(k_head_stats_pair), kPairSmemBytes,
+                    g_pair_ready) != cudaSuccess)
+        return 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2);
     cfg.blockDim = dim3(kHeadThreads);
@@ -530,19 +552,15 @@ int head_stats_pair_max_clusters() {
     cfg.numAttrs = 1;
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, k_head_stats_pair, &cfg) != cudaSuccess) n = 0;
-    cached = n;
+    g_pair_clusters[dev].store(n + 1, std::memory_order_release);
     return n;
 }
 
 cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tmW,
                                    const HeadParams &p, int grid, cudaStream_t s) {
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(k_head_stats_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kPairSmemBytes);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(k_head_stats_pair), kPairSmemBytes,
+                                g_pair_ready);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kHeadThreads);
