@@ -38,8 +38,8 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "1154bab2ebf8d9b6"): 1.0594e9,   # profiles/k_head_stats_pair_llada_first_step.md
-    ("llada_tail_5_masked", "1154bab2ebf8d9b6"): 1.0439e9,       # profiles/k_head_stats_llada_tail5.md
+    ("llada_first_step", "1011354fb1c6ca70"): 1.0599e9,     # profiles/k_head_stats_pair_llada_first_step.md
+    ("llada_tail_5_masked", "1011354fb1c6ca70"): 1.0435e9,  # profiles/k_head_stats_llada_tail5.md
 }
 
 

@@ -21,6 +21,8 @@
  *    records a message for rpd_last_error() (per host thread).  On an error return no
  *    output has been written unless the code is RPD_ERR_CUDA.
  *  - A context is not thread safe; use one context per host thread or serialise calls.
+ *  - Inputs must be finite; with eps = 0 an all-zero hidden row has no defined RMS factor.
+ *    Sums of squares, logits and softmax statistics are fp32 (h^2 must not overflow fp32).
  */
 #ifndef RPD_H_
 #define RPD_H_
