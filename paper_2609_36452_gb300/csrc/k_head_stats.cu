@@ -31,11 +31,30 @@ namespace {
 constexpr uint32_t kTmemCols = 2 * kTileN;
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Work units (row tile m, vocabulary split g) in the order the persistent CTAs take them:
+// row tiles are grouped into bands of `band` tiles; inside a band m runs fastest, then g.
+// The units running at the same time therefore share W tiles (each streamed from HBM once
+// per band) and re-read at most `band` u tiles (kept in L2 while the band runs).  With few
+// row tiles there is a single band and the order is plain (m fastest).
 struct TileWalk {
-    int num_m, num_n, splits, units;
-    __device__ __forceinline__ void unit(int u, int &m, int &n0, int &n1) const {
-        m = u % num_m;
-        const int g = u / num_m;
+    int num_m, num_n, splits, units, band;
+    __device__ __forceinline__ void init(int rows, int tile_rows, int V, int d, int g) {
+        num_m = (rows + tile_rows - 1) / tile_rows;
+        num_n = (V + kTileN - 1) / kTileN;
+        splits = g;
+        units = num_m * splits;
+        const long long tile_bytes = static_cast<long long>(tile_rows) * d * 2;
+        band = static_cast<int>(kBandBytes / tile_bytes);
+        band = max(1, min(num_m, band));
+    }
+    __device__ __forceinline__ void unit(int u, int &m, int &g, int &n0, int &n1) const {
+        const int per_band = band * splits;
+        const int b = u / per_band;
+        const int r = u - b * per_band;
+        const int m0 = b * band;
+        const int in_band = min(band, num_m - m0);
+        m = m0 + r % in_band;
+        g = r / in_band;
         n0 = static_cast<int>((static_cast<long long>(g) * num_n) / splits);
         n1 = static_cast<int>((static_cast<long long>(g + 1) * num_n) / splits);
     }
@@ -125,10 +144,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 
     const int rows = p.meta[kMetaRows];
     TileWalk tw;
-    tw.num_m = (rows + kTileM - 1) / kTileM;
-    tw.num_n = (p.V + kTileN - 1) / kTileN;
-    tw.splits = p.meta[kMetaSplits];
-    tw.units = tw.num_m * tw.splits;
+    tw.init(rows, kTileM, p.V, p.d, p.meta[kMetaSplits]);
     const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (warp == 0) {
@@ -139,8 +155,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             long long fills = 0;
             bool ok = true;
             for (int u = blockIdx.x; ok && u < tw.units; u += gridDim.x) {
-                int m, n0, n1;
-                tw.unit(u, m, n0, n1);
+                int m, g, n0, n1;
+                tw.unit(u, m, g, n0, n1);
                 for (int n = n0; ok && n < n1; ++n) {
                     for (int kb = 0; kb < num_kb; ++kb) {
                         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit_ns)) {
@@ -176,8 +192,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             uint32_t tile_iter = 0;
             bool ok = true;
             for (int u = blockIdx.x; ok && u < tw.units; u += gridDim.x) {
-                int m, n0, n1;
-                tw.unit(u, m, n0, n1);
+                int m, g, n0, n1;
+                tw.unit(u, m, g, n0, n1);
                 for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
                     const uint32_t acc = tile_iter & 1u;
                     const uint32_t acc_phase = (tile_iter >> 1) & 1u;
@@ -224,8 +240,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         uint32_t tile_iter = 0;
         bool ok = true;
         for (int u = blockIdx.x; ok && u < tw.units; u += gridDim.x) {
-            int m, n0, n1;
-            tw.unit(u, m, n0, n1);
+            int m, g, n0, n1;
+            tw.unit(u, m, g, n0, n1);
             const int r = m * kTileM + row_in_tile;
             const bool valid = r < rows;
             const float scale = valid ? p.inv_rms[r] * kLog2e : 0.f;
@@ -256,7 +272,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             }
             if (!ok) break;
             if (valid) {
-                const int g = u / tw.num_m;
                 p.partials[static_cast<size_t>(r) * p.max_splits + g] =
                     make_float4(run_m, run_s, run_t, __int_as_float(run_a));
             }
@@ -338,10 +353,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 
     const int rows = p.meta[kMetaRows];
     TileWalk tw;
-    tw.num_m = (rows + kPairTileM - 1) / kPairTileM;
-    tw.num_n = (p.V + kTileN - 1) / kTileN;
-    tw.splits = p.meta[kMetaSplits];
-    tw.units = tw.num_m * tw.splits;
+    tw.init(rows, kPairTileM, p.V, p.d, p.meta[kMetaSplits]);
     const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (warp == 0) {
@@ -353,8 +365,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             long long fills = 0;
             bool ok = true;
             for (int u = pair; ok && u < tw.units; u += num_pairs) {
-                int m, n0, n1;
-                tw.unit(u, m, n0, n1);
+                int m, g, n0, n1;
+                tw.unit(u, m, g, n0, n1);
                 for (int n = n0; ok && n < n1; ++n) {
                     for (int kb = 0; kb < num_kb; ++kb) {
                         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit_ns)) {
@@ -394,8 +406,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 uint32_t tile_iter = 0;
                 bool ok = true;
                 for (int u = pair; ok && u < tw.units; u += num_pairs) {
-                    int m, n0, n1;
-                    tw.unit(u, m, n0, n1);
+                    int m, g, n0, n1;
+                    tw.unit(u, m, g, n0, n1);
                     for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
                         const uint32_t acc = tile_iter & 1u;
                         const uint32_t acc_phase = (tile_iter >> 1) & 1u;
@@ -444,8 +456,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         uint32_t tile_iter = 0;
         bool ok = true;
         for (int u = pair; ok && u < tw.units; u += num_pairs) {
-            int m, n0, n1;
-            tw.unit(u, m, n0, n1);
+            int m, g, n0, n1;
+            tw.unit(u, m, g, n0, n1);
             const int r = m * kPairTileM + row_in_tile;
             const bool valid = r < rows;
             const float scale = valid ? p.inv_rms[r] * kLog2e : 0.f;
@@ -476,7 +488,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             }
             if (!ok) break;
             if (valid) {
-                const int g = u / tw.num_m;
                 p.partials[static_cast<size_t>(r) * p.max_splits + g] =
                     make_float4(run_m, run_s, run_t, __int_as_float(run_a));
             }

@@ -32,6 +32,7 @@ constexpr int kMaxBatch = 128;
 constexpr int kMaxCanvas = 8192;
 constexpr int kScoreThreads = 1024;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
+constexpr long long kBandBytes = 32ll << 20;       // u tiles a band of head work units re-reads
 
 // Indices into the per-step device metadata words.
 enum MetaIndex : int {

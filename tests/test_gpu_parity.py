@@ -107,6 +107,16 @@ def test_ragged_shapes(d, V, K, N, frac):
     print(rep)
 
 
+def test_many_row_tiles_in_bands():
+    """5100 rows at d = 4096: 20 CTA-pair row tiles (40 single-CTA ones) of 1-2 MB of u each,
+    more than the head kernels keep in one L2 band of work units, so every row of the second
+    band comes from the band-ordered unit walk.  Every output is compared with the oracle."""
+    case = small_case(301, K=5, N=1020, d=4096, V=4100, w_std=0.02)
+    ref, got, rep = run_and_compare(case)
+    assert got["stats"]["n_rows"] == 5 * 1020
+    print(rep)
+
+
 def test_stability_route_with_drops():
     """Flat layer ramp with explicit theta_s: persistence is long and drops small but
     nonzero, so the stability route admits and rejects on the drop penalty."""
