@@ -38,9 +38,9 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "1011354fb1c6ca70"): 1.0599e9,     # profiles/k_head_stats_pair_llada_first_step.md
-    ("llada_tail_5_masked", "1011354fb1c6ca70"): 1.0435e9,  # profiles/k_head_stats_llada_tail5.md
-    ("batched_serving", "3a1e639631c981cf"): 41.42e9,       # profiles/k_head_stats_pair_batched_serving.md
+    ("llada_first_step", "94e34cbf8bd21fb6"): 1.0488e9,     # profiles/k_head_stats_pair_llada_first_step.md
+    ("llada_tail_5_masked", "94e34cbf8bd21fb6"): 1.0435e9,  # profiles/k_head_stats_llada_tail5.md
+    ("batched_serving", "94e34cbf8bd21fb6"): 8.858e9,       # profiles/k_head_stats_pair_batched_serving.md
 }
 
 

@@ -115,6 +115,7 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
         p.meta[kMetaLayer0] = lazy_on ? p.K - 1 : 0;
         p.meta[kMetaRowsTotal] = static_cast<int>(rows);
         p.meta[kMetaLazy] = lazy_on;
+        p.meta[kMetaUnitNext] = 0;
     }
 }
 

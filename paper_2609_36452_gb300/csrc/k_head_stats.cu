@@ -60,6 +60,24 @@ struct TileWalk {
     }
 };
 
+// Work units are claimed at run time from a per-pass counter (meta[kMetaUnitNext]) by the
+// TMA producer, in the walk's order, so the units in flight are always a window of
+// consecutive indices however the CTAs' speeds differ.  The producer passes each claimed
+// index to the MMA issuer and the epilogue warps through a small ring in shared memory
+// (-1: no unit left).
+constexpr int kUnitRing = 4;
+
+struct UnitCursor {
+    int slot = 0;
+    uint32_t phase = 0;
+    __device__ __forceinline__ void advance() {
+        if (++slot == kUnitRing) {
+            slot = 0;
+            phase ^= 1u;
+        }
+    }
+};
+
 // Fold one 32-column chunk (already scaled to log2 units) into the running statistics.
 template <bool kFull>
 __device__ __forceinline__ void fold_chunk(const float (&v)[32], float scale, int col0, int V,
@@ -115,8 +133,11 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     uint64_t *acc_full = bars + 2 * kStages;      // [2] MMA -> epilogue
     uint64_t *acc_empty = bars + 2 * kStages + 2; // [2] epilogue -> MMA
     uint64_t *drain = bars + 2 * kStages + 4;     // [1] MMA completion at exit
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kStages + 5);
+    uint64_t *unit_full = bars + 2 * kStages + 5; // [kUnitRing] producer -> MMA, epilogue
+    uint64_t *unit_empty = unit_full + kUnitRing; // [kUnitRing] MMA, epilogue -> producer
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(unit_empty + kUnitRing);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+    volatile int *unit_ring = abort_flag + 1;     // [kUnitRing] claimed unit indices
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -129,6 +150,10 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&acc_full[i], 1);
             mbar_init(&acc_empty[i], 4);
+        }
+        for (int i = 0; i < kUnitRing; ++i) {
+            mbar_init(&unit_full[i], 1);
+            mbar_init(&unit_empty[i], 1 + 4);  // MMA issuer + 4 epilogue warps
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -154,7 +179,16 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             uint32_t phase = 0;
             long long fills = 0;
             bool ok = true;
-            for (int u = blockIdx.x; ok && u < tw.units; u += gridDim.x) {
+            UnitCursor uc;
+            while (ok) {
+                if (!mbar_wait_bounded(&unit_empty[uc.slot], uc.phase ^ 1u, abort_flag, p.wait_limit_ns))
+                    break;
+                const int claimed = atomicAdd(&p.meta[kMetaUnitNext], 1);
+                const int u = claimed < tw.units ? claimed : -1;
+                unit_ring[uc.slot] = u;
+                mbar_arrive(&unit_full[uc.slot]);
+                uc.advance();
+                if (u < 0) break;
                 int m, g, n0, n1;
                 tw.unit(u, m, g, n0, n1);
                 for (int n = n0; ok && n < n1; ++n) {
@@ -191,7 +225,13 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             uint32_t phase = 0;
             uint32_t tile_iter = 0;
             bool ok = true;
-            for (int u = blockIdx.x; ok && u < tw.units; u += gridDim.x) {
+            UnitCursor uc;
+            while (ok) {
+                if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns)) break;
+                const int u = unit_ring[uc.slot];
+                mbar_arrive(&unit_empty[uc.slot]);
+                uc.advance();
+                if (u < 0) break;
                 int m, g, n0, n1;
                 tw.unit(u, m, g, n0, n1);
                 for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
@@ -239,7 +279,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
         uint32_t tile_iter = 0;
         bool ok = true;
-        for (int u = blockIdx.x; ok && u < tw.units; u += gridDim.x) {
+        UnitCursor uc;
+        while (ok) {
+            if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns)) break;
+            const int u = unit_ring[uc.slot];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&unit_empty[uc.slot]);
+            uc.advance();
+            if (u < 0) break;
             int m, g, n0, n1;
             tw.unit(u, m, g, n0, n1);
             const int r = m * kTileM + row_in_tile;
@@ -320,14 +367,15 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     uint64_t *acc_full = bars + 2 * kPairStages;      // [2]
     uint64_t *acc_empty = bars + 2 * kPairStages + 2; // [2] (used in the even CTA)
     uint64_t *drain = bars + 2 * kPairStages + 4;     // [1]
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kPairStages + 5);
+    uint64_t *unit_full = bars + 2 * kPairStages + 5; // [kUnitRing] even producer -> all others
+    uint64_t *unit_empty = unit_full + kUnitRing;     // [kUnitRing] (used in the even CTA)
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(unit_empty + kUnitRing);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+    volatile int *unit_ring = abort_flag + 1;         // [kUnitRing] claimed unit indices
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const uint32_t rank = cluster_ctarank();  // 0 = even CTA (issues the MMAs), 1 = odd
-    const int pair = blockIdx.x >> 1;
-    const int num_pairs = gridDim.x >> 1;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kPairStages; ++i) {
@@ -337,6 +385,11 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&acc_full[i], 1);
             mbar_init(&acc_empty[i], 8);
+        }
+        for (int i = 0; i < kUnitRing; ++i) {
+            mbar_init(&unit_full[i], 1);
+            // even CTA: its MMA issuer and 4 epilogue warps, the odd producer and 4 epilogue warps
+            mbar_init(&unit_empty[i], 10);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -360,11 +413,36 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         if (lane == 0 && !p.stall) {
             // ------------------------------------------------------- TMA producer (both CTAs)
             const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);
+            const uint32_t unit_full1 = mapa_shared(smem_u32(&unit_full[0]), 1);
+            const uint32_t unit_ring1 = mapa_shared(smem_u32(const_cast<int *>(&unit_ring[0])), 1);
+            const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
             int stage = 0;
             uint32_t phase = 0;
             long long fills = 0;
             bool ok = true;
-            for (int u = pair; ok && u < tw.units; u += num_pairs) {
+            UnitCursor uc;
+            while (ok) {
+                int u;
+                if (rank == 0) {
+                    // claim the next unit and hand it to both CTAs
+                    if (!mbar_wait_bounded_cluster(&unit_empty[uc.slot], uc.phase ^ 1u, abort_flag,
+                                                   p.wait_limit_ns))
+                        break;
+                    const int claimed = atomicAdd(&p.meta[kMetaUnitNext], 1);
+                    u = claimed < tw.units ? claimed : -1;
+                    unit_ring[uc.slot] = u;
+                    st_shared_cluster(unit_ring1 + static_cast<uint32_t>(uc.slot * sizeof(int)), u);
+                    mbar_arrive(&unit_full[uc.slot]);
+                    mbar_arrive_cluster(unit_full1 + static_cast<uint32_t>(uc.slot * sizeof(uint64_t)));
+                } else {
+                    if (!mbar_wait_bounded_cluster(&unit_full[uc.slot], uc.phase, abort_flag,
+                                                   p.wait_limit_ns))
+                        break;
+                    u = unit_ring[uc.slot];
+                    mbar_arrive_cluster(unit_empty0 + static_cast<uint32_t>(uc.slot * sizeof(uint64_t)));
+                }
+                uc.advance();
+                if (u < 0) break;
                 int m, g, n0, n1;
                 tw.unit(u, m, g, n0, n1);
                 for (int n = n0; ok && n < n1; ++n) {
@@ -405,7 +483,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 uint32_t phase = 0;
                 uint32_t tile_iter = 0;
                 bool ok = true;
-                for (int u = pair; ok && u < tw.units; u += num_pairs) {
+                UnitCursor uc;
+                while (ok) {
+                    if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+                        break;
+                    const int u = unit_ring[uc.slot];
+                    mbar_arrive(&unit_empty[uc.slot]);
+                    uc.advance();
+                    if (u < 0) break;
                     int m, g, n0, n1;
                     tw.unit(u, m, g, n0, n1);
                     for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
@@ -453,9 +538,19 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         const int row_in_tile = static_cast<int>(rank) * kPairHalfRows + sub * 32 + lane;
         const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
         const uint32_t acc_empty0 = mapa_shared(smem_u32(&acc_empty[0]), 0);
+        const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
         uint32_t tile_iter = 0;
         bool ok = true;
-        for (int u = pair; ok && u < tw.units; u += num_pairs) {
+        UnitCursor uc;
+        while (ok) {
+            if (!mbar_wait_bounded_cluster(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+                break;
+            const int u = unit_ring[uc.slot];
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive_cluster(unit_empty0 + static_cast<uint32_t>(uc.slot * sizeof(uint64_t)));
+            uc.advance();
+            if (u < 0) break;
             int m, g, n0, n1;
             tw.unit(u, m, g, n0, n1);
             const int r = m * kPairTileM + row_in_tile;

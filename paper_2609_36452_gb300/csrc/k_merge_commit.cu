@@ -110,6 +110,7 @@ __global__ void __launch_bounds__(kBandThreads, 1) k_band(BandParams p) {
         p.meta[kMetaSel] = carry;
         p.meta[kMetaLayer0] = 0;
         p.meta[kMetaRowsTotal] += static_cast<int>(rows);
+        p.meta[kMetaUnitNext] = 0;
     }
 }
 

@@ -45,6 +45,7 @@ enum MetaIndex : int {
     kMetaLayer0 = 6,   // first window layer of the current pass (rows are layer-major)
     kMetaRowsTotal = 7,// rows projected by all passes of this step
     kMetaLazy = 8,     // 1 when this step projects lazily (two passes)
+    kMetaUnitNext = 9, // next head work unit to claim (zeroed before each projection pass)
     kMetaWords = 16
 };
 
