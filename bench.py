@@ -38,9 +38,9 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "94e34cbf8bd21fb6"): 1.0488e9,     # profiles/k_head_stats_pair_llada_first_step.md
-    ("llada_tail_5_masked", "94e34cbf8bd21fb6"): 1.0435e9,  # profiles/k_head_stats_llada_tail5.md
-    ("batched_serving", "94e34cbf8bd21fb6"): 8.858e9,       # profiles/k_head_stats_pair_batched_serving.md
+    ("llada_first_step", "333c34a81c872803"): 1.0505e9,     # profiles/k_head_stats_pair_llada_first_step.md
+    ("llada_tail_5_masked", "333c34a81c872803"): 1.0440e9,  # profiles/k_head_stats_llada_tail5.md
+    ("batched_serving", "333c34a81c872803"): 8.836e9,       # profiles/k_head_stats_pair_batched_serving.md
 }
 
 
@@ -224,6 +224,7 @@ def config_dict(case, R):
             "signal_kappa": case.get("kappa"),
             "projection": "lazy" if "lazy_rows" in case else "all window layers",
             "rows_projected": case.get("lazy_rows", R),
+            "head_tiling": case.get("tiling", "auto (per pass, on the device)"),
             "l2": f"inputs larger than L2: the {2 * case['V'] * case['d'] / 1e9:.2f} GB head is streamed every step"}
 
 
@@ -295,6 +296,10 @@ def run_rpd(args):
     ctx.set_stream(stream)
     ctx.reserve(B, N)
     ctx.set_projection(args.projection)
+    ctx.set_head_tiling(args.tiling)
+    if args.tiling != "auto":
+        case["name"] = case["name"] + "_" + args.tiling
+        case["tiling"] = args.tiling
 
     def step():
         mask.copy_(mask0, non_blocking=True)
@@ -480,6 +485,7 @@ def run_trajectory(args):
     ctx.set_stream(stream)
     ctx.reserve(1, N)
     ctx.set_projection(args.projection)
+    ctx.set_head_tiling(args.tiling)
     peaks = load_peaks()
     hidden_d = torch.empty(K, N, d, dtype=torch.bfloat16, device=dev)
     mask_d = torch.empty(N, dtype=torch.uint8, device=dev)
@@ -568,6 +574,8 @@ def main():
     ap.add_argument("--projection", choices=["all", "lazy", "auto"], default="all",
                     help="window layers projected: all (the step as defined), lazy (earlier "
                          "layers only for band positions), auto (chosen per step on the device)")
+    ap.add_argument("--tiling", choices=["auto", "single", "pair"], default="auto",
+                    help="head contraction tiling (default: chosen per pass on the device)")
     ap.add_argument("--cpu-positions", type=int, default=32)
     ap.add_argument("--ref-positions", type=int, default=8)
     ap.add_argument("--ref-seconds", type=float, default=150.0)

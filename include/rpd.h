@@ -135,6 +135,18 @@ int rpd_reserve(rpd_ctx *ctx, int B, int N);
 #define RPD_PROJECT_AUTO 2
 int rpd_set_projection(rpd_ctx *ctx, int mode);
 
+/* Tiling of the head contraction (no counterpart in the paper; it changes neither the
+ * computed quantities nor, beyond fp32 summation order, their values).  By default
+ * (RPD_TILING_AUTO) the step picks, on the device and per projection pass, the cheaper of:
+ *   RPD_TILING_SINGLE  tiles of 128 rows x 256 vocabulary entries, one CTA each;
+ *   RPD_TILING_PAIR    tiles of 256 rows x 256 entries on CTA pairs (tcgen05 cta_group::2).
+ * Forcing one is for tests and measurements; RPD_TILING_PAIR on a device where no cluster
+ * of two fits falls back to single-CTA tiles. */
+#define RPD_TILING_AUTO 0
+#define RPD_TILING_SINGLE 1
+#define RPD_TILING_PAIR 2
+int rpd_set_head_tiling(rpd_ctx *ctx, int tiling);
+
 /* Diagnostics.  Every wait inside the step's kernels (mbarrier waits of the head kernels) is
  * bounded; when one runs out the kernel stops, drains what it has in flight, frees its
  * tensor memory and latches RPD_ERR_TIMEOUT in rpd_stats.status (the other outputs of that

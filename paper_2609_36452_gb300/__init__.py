@@ -15,7 +15,7 @@ __all__ = [
     "RPD_OK", "RPD_ERR_INVALID_ARGUMENT", "RPD_ERR_NO_HEAD", "RPD_ERR_CUDA",
     "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
-    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
+    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_profile_enable", "rpd_kernel_times",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
@@ -65,6 +65,10 @@ RPD_PROJECT_ALL = 0
 RPD_PROJECT_LAZY = 1
 RPD_PROJECT_AUTO = 2
 PROJECTION_MODES = {"all": RPD_PROJECT_ALL, "lazy": RPD_PROJECT_LAZY, "auto": RPD_PROJECT_AUTO}
+RPD_TILING_AUTO = 0
+RPD_TILING_SINGLE = 1
+RPD_TILING_PAIR = 2
+HEAD_TILINGS = {"auto": RPD_TILING_AUTO, "single": RPD_TILING_SINGLE, "pair": RPD_TILING_PAIR}
 
 
 class RpdError(RuntimeError):
@@ -89,6 +93,7 @@ def _load():
         "rpd_reserve": (i32, [vp, i32, i32]),
         "rpd_set_debug": (i32, [vp, ctypes.POINTER(RpdDebug)]),
         "rpd_set_projection": (i32, [vp, i32]),
+        "rpd_set_head_tiling": (i32, [vp, i32]),
         "rpd_set_wait_limit": (i32, [vp, ctypes.c_int64]),
         "rpd_inject_stall": (i32, [vp]),
         "rpd_step": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
@@ -120,6 +125,7 @@ rpd_set_stream = lib.rpd_set_stream
 rpd_reserve = lib.rpd_reserve
 rpd_set_debug = lib.rpd_set_debug
 rpd_set_projection = lib.rpd_set_projection
+rpd_set_head_tiling = lib.rpd_set_head_tiling
 rpd_set_wait_limit = lib.rpd_set_wait_limit
 rpd_inject_stall = lib.rpd_inject_stall
 rpd_step = lib.rpd_step
@@ -194,6 +200,12 @@ class Rpd:
         if isinstance(mode, bool):
             mode = "lazy" if mode else "all"
         _check(rpd_set_projection(self.handle, PROJECTION_MODES[mode]))
+
+    def set_head_tiling(self, tiling):
+        """Tiling of the head contraction: "auto" (default, chosen per pass on the device),
+        "single" (128-row tiles) or "pair" (256-row tiles on CTA pairs); for tests and
+        measurements."""
+        _check(rpd_set_head_tiling(self.handle, HEAD_TILINGS[tiling]))
 
     def set_wait_limit(self, microseconds: int):
         _check(rpd_set_wait_limit(self.handle, int(microseconds)))

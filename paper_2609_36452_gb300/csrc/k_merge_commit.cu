@@ -102,7 +102,7 @@ __global__ void __launch_bounds__(kBandThreads, 1) k_band(BandParams p) {
     const long long rows = static_cast<long long>(p.K - 1) * carry;
     int mode, splits;
     choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.single_slots, p.pair_slots,
-                       p.hbm_tiles, mode, splits);
+                       p.hbm_tiles, p.tiling, mode, splits);
     if (tid == 0) {
         p.meta[kMetaRows] = static_cast<int>(rows);
         p.meta[kMetaSplits] = splits;

@@ -98,6 +98,7 @@ struct rpd_ctx {
     int32_t *sel_q = nullptr;  // lazy projection: compact indices of the band positions
     int32_t *band_off = nullptr;  // lazy projection: [B+1] each canvas's first band entry
     int projection = RPD_PROJECT_ALL;
+    int tiling = RPD_TILING_AUTO;
     uint64_t wait_limit_ns = kWaitLimitNs;
     bool stall_next = false;  // diagnostics: the next step's head kernels issue no loads
     CUtensorMap tmU{}, tmW{}, tmW_pair{};
@@ -264,7 +265,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         KernelTimer t(c, 0);
         CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
                          num_n, c->max_splits, c->num_sms, pair_slots, hbm_tiles, c->rule.block,
-                         c->projection == RPD_PROJECT_LAZY ? 1 : (lazy ? 2 : 0)};
+                         c->projection == RPD_PROJECT_LAZY ? 1 : (lazy ? 2 : 0), c->tiling};
         e = launch_compact(cp, c->stream);
     }
     if (e != cudaSuccess) return cuda_fail(e, "compaction launch");
@@ -318,6 +319,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             bp.single_slots = c->num_sms;
             bp.pair_slots = pair_slots;
             bp.hbm_tiles = hbm_tiles;
+            bp.tiling = c->tiling;
             for (int b = 0; b < B; ++b) bp.tau[b] = tau[b];
             e = launch_band(bp, c->stream);
         }
@@ -460,6 +462,14 @@ int rpd_set_projection(rpd_ctx *c, int mode) {
     if (mode != RPD_PROJECT_ALL && mode != RPD_PROJECT_LAZY && mode != RPD_PROJECT_AUTO)
         return fail(RPD_ERR_INVALID_ARGUMENT, "unknown projection mode %d", mode);
     c->projection = mode;
+    return RPD_OK;
+}
+
+int rpd_set_head_tiling(rpd_ctx *c, int tiling) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (tiling < RPD_TILING_AUTO || tiling > RPD_TILING_PAIR)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "unknown head tiling %d", tiling);
+    c->tiling = tiling;
     return RPD_OK;
 }
 

@@ -63,6 +63,7 @@ struct CompactParams {
     float hbm_tiles;      // time to stream the head once, in single-CTA tile times
     int block;            // 0: every masked position; > 0: only each canvas's active block
     int lazy;             // 0: all window layers; 1: lazy; 2: lazy when it is estimated cheaper
+    int tiling;           // RPD_TILING_*: head tiling, or 0 to choose per pass
 };
 
 // Band fraction assumed when the device weighs lazy against full projection before the
@@ -93,6 +94,7 @@ struct BandParams {
     float theta_c;
     int num_n_tiles, max_splits, single_slots, pair_slots;
     float hbm_tiles;
+    int tiling;
     float tau[kMaxBatch];
 };
 

@@ -202,7 +202,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     if (e == cudaSuccess) {
         CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n, splits,
                          dev->num_sms, pair_slots, head_stream_in_tiles(V, d, dev->num_sms),
-                         rule.block, 0};
+                         rule.block, 0, RPD_TILING_AUTO};
         e = launch_compact(cp, stream);
     }
     if (e == cudaSuccess) {

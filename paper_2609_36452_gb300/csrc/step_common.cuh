@@ -21,10 +21,12 @@ __device__ __forceinline__ int warp_inclusive_scan(int v, int lane) {
 // 256 rows on `pair_slots` pairs) take the vocabulary split count G minimising
 // waves * n-tiles-per-unit (smallest G on ties); estimate the time as the larger of the MMA
 // work of the busiest slot and the head streaming time scaled by the vocabulary share of the
-// largest split, in single-tile units; keep the cheaper tiling.  Called by every thread of
-// the CTA; the result (and the returned estimate) is valid in thread 0.
+// largest split, in single-tile units; keep the cheaper tiling, or the one `force` names
+// (RPD_TILING_*; CTA pairs only where they are available).  Called by every thread of the
+// CTA; the result (and the returned estimate) is valid in thread 0.
 __device__ float choose_head_tiling(long long rows, int num_n, int max_splits, int single_slots,
-                                    int pair_slots, float hbm_tiles, int &mode, int &splits) {
+                                    int pair_slots, float hbm_tiles, int force, int &mode,
+                                    int &splits) {
     __shared__ unsigned long long best1, best2;
     const int tid = threadIdx.x;
     const int gmax = min(num_n, max_splits);
@@ -63,7 +65,7 @@ __device__ float choose_head_tiling(long long rows, int num_n, int max_splits, i
             const float per2 = static_cast<float>((num_n + g2 - 1) / g2);
             const float est2 = fmaxf(kPairTileCost * static_cast<float>(best2 >> 20),
                                      hbm_tiles * per2 * g2 / num_n);
-            if (est2 < est1) {
+            if (force == RPD_TILING_PAIR || (force != RPD_TILING_SINGLE && est2 < est1)) {
                 mode = 2;
                 splits = g2;
                 est = est2;

@@ -107,6 +107,28 @@ def test_ragged_shapes(d, V, K, N, frac):
     print(rep)
 
 
+@pytest.mark.parametrize("tiling", ["single", "pair"])
+@pytest.mark.parametrize("d,V,K,N,frac", [
+    (256, 4100, 3, 100, 1.0),    # 300 rows: ragged last row tile of either tiling
+    (4096, 1280, 3, 50, 1.0),    # 150 rows, 64 K-blocks
+    (200, 1000, 2, 77, 0.7),     # ragged K-block and vocabulary tile, ~108 rows
+    (128, 4100, 5, 300, 1.0),    # 1500 rows: 12 single / 6 pair row tiles
+    (64, 512, 4, 128, 1.0),      # 512 rows: whole row tiles only
+])
+def test_head_tilings_match_oracle(tiling, d, V, K, N, frac):
+    """Both head tilings, forced, on the same inputs; each is compared with the oracle
+    element by element."""
+    case = small_case(11 + d + V + K, K=K, N=N, d=d, V=V, w_std=0.08, mask_frac=frac)
+    runner = GpuRunner(case["W"], case["g"], K, case["eps"], rule=case["rule"])
+    try:
+        runner.ctx.set_head_tiling(tiling)
+        got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+    finally:
+        runner.close()
+    ref = oracle_step(case)
+    print(compare_step(ref, got))
+
+
 def test_many_row_tiles_in_bands():
     """5100 rows at d = 4096: 20 CTA-pair row tiles (40 single-CTA ones) of 1-2 MB of u each,
     more than the head kernels keep in one L2 band of work units, so every row of the second
