@@ -165,7 +165,8 @@ int rpd_set_debug(rpd_ctx *ctx, const rpd_debug *debug);
  *              each canvas position (the final layer last).  Rows of unmasked
  *              positions are never read.
  *   mask       [N] uint8, device, in/out: 1 = masked.  Committed positions are set to 0.
- *   N          canvas length, 0 <= N <= 8192 (N = 0 is a no-op).
+ *   N          canvas length, 0 <= N <= 8192 (N = 0 is a no-op; N > 8192:
+ *              RPD_ERR_UNSUPPORTED).
  *   tau        theta_h, 0 < tau <= 1 and tau > theta_c.
  *   budget     beta in nats, >= 0 (may be +inf).
  *   out_commit [N] uint8, device: 1 where committed this step, 0 elsewhere.
@@ -179,9 +180,10 @@ int rpd_step(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau, 
 /* B independent canvases of N positions in one step; the head is read once for all.
  *   hidden [K][B][N][d] bf16 device; mask, out_commit, out_token [B][N] device;
  *   tau, budget [B] HOST arrays (per-canvas theta_h and beta); out_stats [B] device.
- * Requires 1 <= B <= 128.  Canvases of different lengths are padded to a common N with mask
- * 0: unmasked positions are never projected, scored, counted in E_i or committed, so each
- * canvas's result is that of its unpadded length. */
+ * Requires 1 <= B <= 128 (B > 128 or N > 8192: RPD_ERR_UNSUPPORTED).  Canvases of
+ * different lengths are padded to a common N with mask 0: unmasked positions are never
+ * projected, scored, counted in E_i or committed, so each canvas's result is that of its
+ * unpadded length. */
 int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int N,
                      const float *tau, const float *budget, uint8_t *out_commit,
                      int32_t *out_token, rpd_stats *out_stats);

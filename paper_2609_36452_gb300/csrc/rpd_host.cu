@@ -236,7 +236,8 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
              const float *budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
     if (!c->W || !c->g) return fail(RPD_ERR_NO_HEAD, "rpd_set_head has not been called");
-    if (B < 1 || B > kMaxBatch) return fail(RPD_ERR_INVALID_ARGUMENT, "B must be in [1, %d]", kMaxBatch);
+    if (B < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "B must be >= 1");
+    if (B > kMaxBatch) return fail(RPD_ERR_UNSUPPORTED, "B must be <= %d", kMaxBatch);
     if (N < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be >= 0");
     if (N > kMaxCanvas) return fail(RPD_ERR_UNSUPPORTED, "N must be <= %d", kMaxCanvas);
     if (!tau || !budget) return fail(RPD_ERR_INVALID_ARGUMENT, "null tau/budget");
@@ -452,8 +453,9 @@ int rpd_set_stream(rpd_ctx *c, void *stream) {
 
 int rpd_reserve(rpd_ctx *c, int B, int N) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
-    if (B < 1 || B > kMaxBatch || N < 1 || N > kMaxCanvas)
-        return fail(RPD_ERR_INVALID_ARGUMENT, "reserve: B in [1,%d], N in [1,%d]", kMaxBatch, kMaxCanvas);
+    if (B < 1 || N < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "reserve: B and N must be >= 1");
+    if (B > kMaxBatch || N > kMaxCanvas)
+        return fail(RPD_ERR_UNSUPPORTED, "reserve: B <= %d, N <= %d", kMaxBatch, kMaxCanvas);
     return ensure_scratch(c, B, N);
 }
 
@@ -509,7 +511,8 @@ int rpd_step_batched(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N
 int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float tau, float budget,
                   uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
-    if (N < 0 || N > kMaxCanvas) return fail(RPD_ERR_INVALID_ARGUMENT, "N out of range");
+    if (N < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be >= 0");
+    if (N > kMaxCanvas) return fail(RPD_ERR_UNSUPPORTED, "N must be <= %d", kMaxCanvas);
     if (N == 0) return run_step(c, nullptr, nullptr, 1, 0, &tau, &budget, nullptr, nullptr, nullptr);
     if (!hidden || !mask || !out_commit || !out_token || !out_stats)
         return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");

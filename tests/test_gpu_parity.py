@@ -527,3 +527,43 @@ def test_exact_argmax_tie_takes_lowest_token():
     assert np.all(ref.layer_argmax == lo) and np.all(ref.layer_gap == 0.0)
     assert np.all(got["layer_argmax"] == lo)
     assert np.all(got["token"][got["commit"] == 1] == lo)
+
+
+# ------------------------------------------------------------------ window and canvas limits
+
+@pytest.mark.parametrize("K,N,rule", [(16, 96, "llada"), (14, 96, "dream"), (64, 40, "llada")])
+def test_paper_windows_and_largest_window(K, N, rule):
+    """The windows the paper projects (the last 16 layers of LLaDA, the last 14 of Dream;
+    App. A.6) and the largest the library accepts (K = 64).  A flat layer ramp keeps the
+    argmax through many layers, so persistence reaches k_max and stability admissions occur."""
+    case = small_case(5 + K + N, K=K, N=N, d=256, V=1024, a=torch.ones(K), rule=rule)
+    ref, got, rep = run_and_compare(case)
+    assert np.max(got["persist"][ref.masked]) >= 6
+    print(rep)
+
+
+def test_largest_canvas():
+    """One canvas of N = 8192 positions (the largest accepted), half of them masked: the
+    widest instantiation of the score/commit kernel.  N = 8193 is refused before any work."""
+    case = small_case(8201, K=2, N=8192, d=256, V=1024, mask_frac=0.5)
+    ref, got, rep = run_and_compare(case)
+    assert got["stats"]["n_masked"] == int(case["mask"].sum())
+    print(rep)
+    import paper_2609_36452_gb300 as rpd
+    dev = torch.device("cuda:0")
+    ctx = rpd.Rpd(256, 1024, 2)
+    try:
+        ctx.set_head(case["W"].to(dev), case["g"].to(dev))
+        n = 8193
+        h = torch.zeros(2, n, 256, dtype=torch.bfloat16, device=dev)
+        m = torch.ones(n, dtype=torch.uint8, device=dev)
+        c = torch.full((n,), 7, dtype=torch.uint8, device=dev)
+        t = torch.zeros(n, dtype=torch.int32, device=dev)
+        s = torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev)
+        with pytest.raises(rpd.RpdError) as e:
+            ctx.step(h, m, 0.9, 1.0, c, t, s)
+        assert e.value.code == rpd.RPD_ERR_UNSUPPORTED
+        torch.cuda.synchronize(dev)
+        assert torch.all(c == 7) and torch.all(m == 1)
+    finally:
+        ctx.close()
