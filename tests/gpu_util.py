@@ -10,7 +10,7 @@ def bits(t: torch.Tensor) -> np.ndarray:
     return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
 
 
-class GpuRunner:
+class DeviceRunner:
     """Context + head on cuda:0; runs single or batched steps with every debug output."""
 
     def __init__(self, W: torch.Tensor, g: torch.Tensor, K: int, eps: float = 1e-6, rule="llada"):

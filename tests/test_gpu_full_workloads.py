@@ -15,7 +15,7 @@ import torch
 
 import workloads as WL
 from oracle import rpd_oracle as O
-from tests.gpu_util import GpuRunner, bits
+from tests.gpu_util import DeviceRunner, bits
 from tests.parity import DELTA, compare_rows, compare_step, replay_commit_rule
 
 pytestmark = pytest.mark.gpu
@@ -40,7 +40,7 @@ def oracle_rows(hidden_rows, g, W, eps):
 def test_batched_serving_full():
     case = WL.batched_serving(seed=5)
     K, B, N = case["K"], case["B"], case["N"]
-    runner = GpuRunner(case["W"], case["g"], K, case["eps"], rule="llada")
+    runner = DeviceRunner(case["W"], case["g"], K, case["eps"], rule="llada")
     try:
         outs = runner.step_batched(case["hidden"], case["mask"], case["tau"], case["budget"])
     finally:
@@ -88,7 +88,7 @@ def test_llada_trajectory(traj_head):
     K, N, V = 4, 256, WL.LLADA_V
     gen = torch.Generator().manual_seed(4004)
     targets = torch.randint(0, V, (N,), generator=gen)
-    runner = GpuRunner(W, g, K, 1e-6, rule="llada")
+    runner = DeviceRunner(W, g, K, 1e-6, rule="llada")
     mask = torch.ones(N, dtype=torch.uint8)
     checked = []
     steps = []

@@ -12,7 +12,7 @@ import torch
 
 import workloads as WL
 from oracle import rpd_oracle as O
-from tests.gpu_util import GpuRunner, bits
+from tests.gpu_util import DeviceRunner, bits
 from tests.parity import compare_block_step, compare_step
 
 pytestmark = pytest.mark.gpu
@@ -50,7 +50,7 @@ def small_case(seed, K=3, N=64, d=256, V=4096, w_std=0.08, sigma=None, flip=0.1,
 
 
 def run_and_compare(case, rule=None, tau=None, budget=None, mask=None):
-    runner = GpuRunner(case["W"], case["g"], case["K"], case["eps"],
+    runner = DeviceRunner(case["W"], case["g"], case["K"], case["eps"],
                        rule=case["rule"] if rule is None else rule)
     try:
         m = case["mask"] if mask is None else mask
@@ -119,7 +119,7 @@ def test_head_tilings_match_oracle(tiling, d, V, K, N, frac):
     """Both head tilings, forced, on the same inputs; each is compared with the oracle
     element by element."""
     case = small_case(11 + d + V + K, K=K, N=N, d=d, V=V, w_std=0.08, mask_frac=frac)
-    runner = GpuRunner(case["W"], case["g"], K, case["eps"], rule=case["rule"])
+    runner = DeviceRunner(case["W"], case["g"], K, case["eps"], rule=case["rule"])
     try:
         runner.ctx.set_head_tiling(tiling)
         got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
@@ -167,7 +167,7 @@ def test_fallback_window_counts_masked_positions():
 
 def test_empty_and_single_masks():
     case = small_case(45, K=3, N=40)
-    runner = GpuRunner(case["W"], case["g"], 3)
+    runner = DeviceRunner(case["W"], case["g"], 3)
     try:
         none = torch.zeros(40, dtype=torch.uint8)
         got = runner.step(case["hidden"], none, 0.9, 1.0)
@@ -200,7 +200,7 @@ def test_batched_matches_per_canvas_oracle():
         hidden[:, b] = cv.hidden
         masks[b] = WL.uniform_fraction_mask(N, [1.0, 0.5, 0.0, 0.9][b], 700 + b)
     taus, budgets = [0.9, 0.8, 0.9, 0.95], [1.0, 3.0, 1.0, 0.5]
-    runner = GpuRunner(W, g, K)
+    runner = DeviceRunner(W, g, K)
     try:
         outs = runner.step_batched(hidden, masks, taus, budgets)
     finally:
@@ -214,7 +214,7 @@ def test_batched_matches_per_canvas_oracle():
 
 def test_host_entry_point_matches_device():
     case = small_case(61, K=3, N=64)
-    runner = GpuRunner(case["W"], case["g"], 3)
+    runner = DeviceRunner(case["W"], case["g"], 3)
     try:
         dev = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
         hid = case["hidden"].contiguous().pin_memory()
@@ -236,7 +236,7 @@ def test_host_entry_point_matches_device():
 
 def test_repeat_is_bit_identical():
     case = small_case(71, K=4, N=200, d=512, V=3000)
-    runner = GpuRunner(case["W"], case["g"], 4)
+    runner = DeviceRunner(case["W"], case["g"], 4)
     try:
         a = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
         b = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
@@ -313,7 +313,7 @@ def test_rpd_block_matches_oracle(block, prefix):
     mask = case["mask"].clone()
     mask[:prefix] = 0
     rule = block_rule(block)
-    runner = GpuRunner(case["W"], case["g"], case["K"], case["eps"], rule=rule)
+    runner = DeviceRunner(case["W"], case["g"], case["K"], case["eps"], rule=rule)
     try:
         got = runner.step(case["hidden"], mask, case["tau"], case["budget"])
     finally:
@@ -336,7 +336,7 @@ def test_rpd_block_batched_canvases():
     masks[1, :33] = 0   # canvas 1: active block starts at 32
     masks[2, :] = 0     # canvas 2: nothing masked
     rule = block_rule(32)
-    runner = GpuRunner(W, g, K, rule=rule)
+    runner = DeviceRunner(W, g, K, rule=rule)
     try:
         outs = runner.step_batched(hidden, masks, [0.9] * B, [1.0] * B)
     finally:
@@ -353,7 +353,7 @@ def test_rpd_block_llada_first_step_full(llada_head):
     W, g = llada_head
     case = WL.llada_first_step(seed=2, W=W, g=g)
     rule = block_rule(32)
-    runner = GpuRunner(W, g, case["K"], case["eps"], rule=rule)
+    runner = DeviceRunner(W, g, case["K"], case["eps"], rule=rule)
     try:
         got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
     finally:
@@ -369,7 +369,7 @@ def test_rpd_block_llada_first_step_full(llada_head):
 def run_lazy_and_eager(case, rule=None, tau=None, budget=None):
     outs = {}
     for lazy in (False, True):
-        runner = GpuRunner(case["W"], case["g"], case["K"], case["eps"],
+        runner = DeviceRunner(case["W"], case["g"], case["K"], case["eps"],
                            rule=case["rule"] if rule is None else rule)
         runner.ctx.set_projection(lazy)
         try:
@@ -436,7 +436,7 @@ def test_auto_projection_picks_per_step(llada_head):
     for mask, expect_lazy in ((case["mask"], True), (tail, False)):
         outs = {}
         for mode in ("all", "auto"):
-            runner = GpuRunner(W, g, case["K"], case["eps"], rule="llada")
+            runner = DeviceRunner(W, g, case["K"], case["eps"], rule="llada")
             runner.ctx.set_projection(mode)
             try:
                 outs[mode] = runner.step(case["hidden"], mask, case["tau"], case["budget"])
@@ -471,7 +471,7 @@ def test_batched_heterogeneous_lengths():
         hidden[:, b, nb:] = 0          # padding rows carry nothing
         masks[b, :nb] = WL.uniform_fraction_mask(nb, 0.8, 950 + b)
     taus, budgets = [0.9, 0.85, 0.9], [1.0, 2.0, 0.5]
-    runner = GpuRunner(W, g, K)
+    runner = DeviceRunner(W, g, K)
     try:
         outs = runner.step_batched(hidden, masks, taus, budgets)
     finally:
@@ -494,7 +494,7 @@ def test_stalled_head_reports_timeout_and_context_recovers(N, K):
     same context is correct again."""
     import paper_2609_36452_gb300 as rpd
     case = small_case(301 + N, K=K, N=N)
-    runner = GpuRunner(case["W"], case["g"], K)
+    runner = DeviceRunner(case["W"], case["g"], K)
     try:
         runner.ctx.set_wait_limit(20000)          # 20 ms
         runner.ctx.inject_stall()
@@ -518,7 +518,7 @@ def test_exact_argmax_tie_takes_lowest_token():
     cv = WL.make_hidden(W, K, N, 98, torch.full((N,), 3.0), WL.calibrated_sigma(V, d, 0.08, 3.0),
                         targets=targets)
     mask = torch.ones(N, dtype=torch.uint8)
-    runner = GpuRunner(W, g, K)
+    runner = DeviceRunner(W, g, K)
     try:
         got = runner.step(cv.hidden, mask, 0.9, 1.0)
     finally:
