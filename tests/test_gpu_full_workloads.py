@@ -4,8 +4,9 @@
   (~32k projected rows).  Sampled positions of every canvas are projected by the oracle and
   compared score by score; the commitment of every canvas is checked by replaying the
   oracle's rule on the GPU's own scores (a property that holds at any size).
-* Decode trajectory at the LLaDA-8B head shape: every step's invariants, and the full oracle
-  at the first, a middle and the last step.
+* Decode trajectory at the LLaDA-8B head shape: at every step the invariants, the commit
+  rule replayed on the GPU's scores and two sampled positions against the oracle; the full
+  oracle at the first, a middle and the last step.
 """
 import math
 
@@ -108,6 +109,26 @@ def test_llada_trajectory(traj_head):
     finally:
         runner.close()
     assert int(mask.sum()) <= 0.02 * N, "trajectory did not finish within 64 steps"
+    # every step: the commit rule replayed on the GPU's own scores, and two sampled masked
+    # positions projected by the oracle (one fp64 projection for all sampled rows)
+    rule = O.RULES["llada"]
+    pick = np.random.default_rng(404)
+    samples = []
+    for t, (cv, m, got) in enumerate(steps):
+        masked = m.numpy().astype(bool)
+        exp, cand, near = replay_commit_rule(got, masked, 0.9, 1.0, rule, K)
+        diff = np.nonzero(exp != got["commit"])[0]
+        if near:
+            assert np.all(diff >= min(near)), (t, diff[:10], sorted(near)[:5])
+        else:
+            assert len(diff) == 0, (t, diff[:10])
+        idx = np.nonzero(masked)[0]
+        samples += [(t, int(i)) for i in pick.choice(idx, size=min(2, len(idx)), replace=False)]
+    rows = torch.stack([steps[t][0].hidden[:, i] for t, i in samples])     # [P][K][d]
+    readouts = dict(zip(samples, oracle_rows(rows, g, W, 1e-6)))
+    for t, (cv, m, got) in enumerate(steps):
+        mine = [i for tt, i in samples if tt == t]
+        compare_rows({i: readouts[(t, i)] for i in mine}, got, mine, K)
     for t in sorted({0, len(steps) // 2, len(steps) - 1}):
         cv, m, got = steps[t]
         ref = O.rpd_step(bits(cv.hidden), m.numpy(), bits(g), bits(W), 1e-6, 0.9, 1.0, "llada")
