@@ -4,8 +4,9 @@ Default workload (N=1): the LLaDA-8B-shaped first step - batch 1, a 256-position
 all masked, K=4 window layers, d=4096, V=126464 (1024 projected rows), tau 0.9, budget
 1.0 - with synthetic seeded inputs (the calibrated hidden-state recipe of ``workloads``).
 One "step" is one rpd_step call: gather + RMSNorm prologue, tcgen05 head statistics,
-split merge, scoring/scan/commit.  The canvas mask is restored before each step (a
-256-byte device copy) so every step sees the same workload.
+split merge, scoring/scan/commit.  The step clears committed positions of its mask, so
+every timed step reads its own copy of the input mask, written before the timed region:
+each step sees the same workload and the timed region holds nothing but the steps.
 
 Metric: commit steps/s (and rows/s).  Under torchrun each rank runs its own canvas
 (weak scaling, no collective on the data path; a barrier and a max-reduce of the timer
@@ -285,7 +286,11 @@ def run_rpd(args):
     g = case["g"].to(dev)
     hidden = case["hidden"].to(dev).contiguous()
     mask0 = case["mask"].to(dev)
-    mask = mask0.clone()
+    # The step clears committed positions of its mask in place.  Every step of a timed pass
+    # gets its own copy of the input mask, written before the pass starts, so the timed
+    # region holds the steps alone (no reset copies between them).
+    n_masks = max(args.steps, args.warmup)
+    masks = mask0.unsqueeze(0).repeat(n_masks, *([1] * mask0.dim())).contiguous()
     commit = torch.zeros(B, N, dtype=torch.uint8, device=dev)
     token = torch.full((B, N), -1, dtype=torch.int32, device=dev)
     stats = torch.zeros(B, rpd.STATS_WORDS, dtype=torch.int32, device=dev)
@@ -301,8 +306,12 @@ def run_rpd(args):
         case["name"] = case["name"] + "_" + args.tiling
         case["tiling"] = args.tiling
 
-    def step():
-        mask.copy_(mask0, non_blocking=True)
+    def refill_masks():
+        masks.copy_(mask0.unsqueeze(0).expand_as(masks))
+        torch.cuda.synchronize(dev)
+
+    def step(i):
+        mask = masks[i % n_masks]
         if B == 1:
             ctx.step(hidden, mask.reshape(N), case["tau"], case["budget"], commit[0], token[0], stats[0])
         else:
@@ -324,8 +333,9 @@ def run_rpd(args):
     sampler = ClockSampler(local) if rank == 0 else None
     if sampler:
         sampler.start()
-    for _ in range(args.warmup):
-        step()
+    refill_masks()
+    for i in range(args.warmup):
+        step(i)
     torch.cuda.synchronize(dev)
     st = [rpd.stats_dict(stats[b].cpu()) for b in range(B)]
     assert all(x["status"] == 0 for x in st), st
@@ -343,23 +353,25 @@ def run_rpd(args):
 
     # Timed pass 1: the step time (no per-kernel events, which would serialise the
     # programmatic-dependent-launch overlap between the step's kernels).
+    refill_masks()
     barrier()
     torch.cuda.synchronize(dev)
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
-        step()
+    for i in range(args.steps):
+        step(i)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
     ms_local = e0.elapsed_time(e1)
     # Timed pass 2: the same K steps with CUDA events around every launch on the context's
     # stream, for per-kernel durations (the roofline of the dominant kernel).
+    refill_masks()
     ctx.kernel_times(reset=True)
     ctx.profile(True)
-    for _ in range(args.steps):
-        step()
+    for i in range(args.steps):
+        step(i)
     torch.cuda.synchronize(dev)
     ctx.profile(False)
     clocks = sampler.stop() if sampler else None
