@@ -51,7 +51,7 @@ def small_case(seed, K=3, N=64, d=256, V=4096, w_std=0.08, sigma=None, flip=0.1,
 
 def run_and_compare(case, rule=None, tau=None, budget=None, mask=None):
     runner = DeviceRunner(case["W"], case["g"], case["K"], case["eps"],
-                       rule=case["rule"] if rule is None else rule)
+                          rule=case["rule"] if rule is None else rule)
     try:
         m = case["mask"] if mask is None else mask
         got = runner.step(case["hidden"], m, case["tau"] if tau is None else tau,
@@ -212,6 +212,45 @@ def test_batched_matches_per_canvas_oracle():
     assert outs[2]["stats"]["n_masked"] == 0
 
 
+def test_largest_batch():
+    """B = 128 canvases (the most one call accepts) of 24 positions, with masked counts from
+    0 and 1 up to all 24 and per-canvas thresholds; every canvas against its own oracle
+    step.  B = 129 is refused."""
+    K, N, d, V, B = 2, 24, 128, 1024, 128
+    W, g = WL.make_head(V, d, 57, w_std=0.3)
+    hidden = torch.empty(K, B, N, d, dtype=torch.bfloat16)
+    masks = torch.zeros(B, N, dtype=torch.uint8)
+    gen = torch.Generator().manual_seed(5700)
+    for b in range(B):
+        cv = WL.make_hidden(W, K, N, 5800 + b, WL.u_profile(N, 0.5, 3.0),
+                              WL.calibrated_sigma(V, d, 0.3, 3.0), flip_frac=0.1)
+        hidden[:, b] = cv.hidden
+        n_masked = b % (N + 1)                      # 0, 1, ..., N, 0, 1, ...
+        masks[b, torch.randperm(N, generator=gen)[:n_masked]] = 1
+    taus = [0.9 if b % 3 else 0.7 for b in range(B)]
+    budgets = [float(b % 5) for b in range(B)]
+    runner = DeviceRunner(W, g, K)
+    try:
+        outs = runner.step_batched(hidden, masks, taus, budgets)
+        import paper_2609_36452_gb300 as rpd
+        dev = torch.device("cuda:0")
+        big = torch.ones(B + 1, N, dtype=torch.uint8, device=dev)
+        h = torch.zeros(K, B + 1, N, d, dtype=torch.bfloat16, device=dev)
+        c = torch.zeros(B + 1, N, dtype=torch.uint8, device=dev)
+        t = torch.zeros(B + 1, N, dtype=torch.int32, device=dev)
+        s = torch.zeros(B + 1, rpd.STATS_WORDS, dtype=torch.int32, device=dev)
+        with pytest.raises(rpd.RpdError) as e:
+            runner.ctx.step_batched(h, big, [0.9] * (B + 1), [1.0] * (B + 1), c, t, s)
+        assert e.value.code == rpd.RPD_ERR_UNSUPPORTED
+    finally:
+        runner.close()
+    for b in range(B):
+        ref = O.rpd_step(bits(hidden[:, b]), masks[b].numpy(), bits(g), bits(W), 1e-6, taus[b],
+                         budgets[b], "llada")
+        compare_step(ref, outs[b])
+        assert (outs[b]["stats"]["n_committed"] >= 1) == (b % (N + 1) > 0)
+
+
 def test_host_entry_point_matches_device():
     case = small_case(61, K=3, N=64)
     runner = DeviceRunner(case["W"], case["g"], 3)
@@ -370,7 +409,7 @@ def run_lazy_and_eager(case, rule=None, tau=None, budget=None):
     outs = {}
     for lazy in (False, True):
         runner = DeviceRunner(case["W"], case["g"], case["K"], case["eps"],
-                           rule=case["rule"] if rule is None else rule)
+                              rule=case["rule"] if rule is None else rule)
         runner.ctx.set_projection(lazy)
         try:
             outs[lazy] = runner.step(case["hidden"], case["mask"], case["tau"] if tau is None else tau,
