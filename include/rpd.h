@@ -53,7 +53,7 @@ typedef struct rpd_rule {
     float w;        /* weight of the confidence-drop penalty (Eq. 4), >= 0 */
     int32_t k_max;  /* cap on prediction persistence (Eq. 4), >= 1 */
     int32_t window; /* fallback window W: first W masked positions (§3.2), >= 1 */
-    int32_t block;  /* 0: full RPD (§3.2).  > 0: RPD-block (§3.2 "Variants", App. A.6):
+    int32_t block;  /* 0: full RPD (§3.2).  > 0: RPD-block (the variant of §3.2, App. A.6):
                        only the active block - the first run of `block` positions (32 in
                        the paper) that still holds a masked position - is projected and
                        scored; every candidate in it is committed (no entropy budget;
@@ -117,7 +117,7 @@ int rpd_set_stream(rpd_ctx *ctx, void *stream);
  * allocate nothing.  Steps grow scratch on demand otherwise (synchronising the device). */
 int rpd_reserve(rpd_ctx *ctx, int B, int N);
 
-/* How the window layers are projected (App. A.6, "Layerwise projection").
+/* How the window layers are projected (App. A.6, the layerwise projection).
  *   RPD_PROJECT_ALL (default): every window layer of every scored position, in one pass over
  *     the head.
  *   RPD_PROJECT_LAZY: a first pass projects the final layer of every scored position; a second

@@ -87,8 +87,8 @@ def f64_to_bf16_rne(x) -> np.ndarray:
 
 
 # ----------------------------------------------------------------------------------------
-# Layerwise projection (§2.2 logit lens; App. A.2 "Intermediate-layer readout"; App. A.6
-# "Layerwise projection": final normalisation + output head on masked positions only)
+# Layerwise projection (§2.2 logit lens; App. A.2, the readout of intermediate layers; App.
+# A.6, the projection as implemented: final normalisation + output head on masked positions only)
 # ----------------------------------------------------------------------------------------
 
 def rms_factor(h_bits, eps: float) -> np.ndarray:
@@ -358,7 +358,7 @@ def active_block(masked, block: int):
 
 def rpd_block_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, rule,
                    block: int = 32) -> StepResult:
-    """RPD-block (§3.2 "Variants", App. A.6): the candidate selection of Eq. 5 applied within
+    """RPD-block (the variant of §3.2, App. A.6): the candidate selection of Eq. 5 applied within
     the active block of ``block`` positions, no cumulative-entropy budget (every candidate of
     the block is committed), and, when no candidate passes, the most confident masked
     position of the active block (leftmost on ties)."""

@@ -1,4 +1,4 @@
-"""Pins of the RPD-block oracle (§3.2 "Variants", App. A.6 "RPD-block")."""
+"""Pins of the RPD-block oracle (the block variant of §3.2 and App. A.6)."""
 import json
 import math
 import os
