@@ -216,6 +216,18 @@ def run_reference(args):
     print(json.dumps(out))
 
 
+def launches_per_step(case, args) -> int:
+    """Kernels one rpd_step / rpd_step_batched call launches: the compaction; per projection
+    pass gather/norm, both head tilings (the one not chosen returns at once) and the merge;
+    the band selection before a second (lazy) pass; and score/commit, which the last merge
+    performs itself for a single canvas of at most 2048 positions."""
+    B = case.get("B", 1)
+    K, N = case["K"], case["N"]
+    second_pass = args.projection == "lazy" or (args.projection == "auto" and K > 1 and K * B * N > 256)
+    fused_score = B == 1 and N <= 2048
+    return 1 + 4 * (2 if second_pass else 1) + (1 if second_pass else 0) + (0 if fused_score else 1)
+
+
 def config_dict(case, R):
     B = case.get("B", 1)
     rule = case["rule"]
@@ -467,7 +479,7 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
         "kernel_timing": "per step; second timed pass of the same steps with CUDA events around each launch",
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 6 * args.steps,  # compact, gather/norm, two head tilings (one returns at once), merge, score/commit
+        "gpu_launches": launches_per_step(case, args) * args.steps,
         "clocks": clocks,
         "last_step_stats": st,
     }

@@ -199,8 +199,10 @@ int rpd_step_host(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float 
 /* Per-kernel timing with CUDA events recorded on the context's stream around every
  * launch while enabled.  rpd_kernel_times synchronises the recorded events and returns,
  * for each of the RPD_NUM_KERNELS kernels (gather/norm, head statistics, merge,
- * score/commit; the compaction kernel is counted with gather/norm), the summed
- * milliseconds and the launch count since the last reset; reset clears them. */
+ * score/commit; the compaction kernel is counted with gather/norm, and for a single canvas
+ * of at most 2048 positions score/commit runs inside the step's last merge and is counted
+ * with it), the summed milliseconds and the launch count since the last reset; reset
+ * clears them. */
 #define RPD_NUM_KERNELS 4
 int rpd_profile_enable(rpd_ctx *ctx, int enable);
 int rpd_kernel_times(rpd_ctx *ctx, double *ms /*[RPD_NUM_KERNELS]*/,

@@ -116,6 +116,7 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
         p.meta[kMetaRowsTotal] = static_cast<int>(rows);
         p.meta[kMetaLazy] = lazy_on;
         p.meta[kMetaUnitNext] = 0;
+        p.meta[kMetaMergeDone] = 0;
     }
 }
 

@@ -31,9 +31,11 @@
 namespace rpd {
 namespace {
 
+constexpr int kMergeThreads = 256;
+
 // Grid-wide merge of the current projection pass (every row of every canvas).
-__global__ void __launch_bounds__(256) k_merge(MergeArgs mg, const int32_t *meta,
-                                               const int32_t *sel_list) {
+__global__ void __launch_bounds__(kMergeThreads) k_merge(MergeArgs mg, const int32_t *meta,
+                                                         const int32_t *sel_list) {
     pdl_trigger();  // successors may launch now; they wait for this grid before reading
     pdl_wait();
     merge_pass_rows(mg, meta, sel_list, 0, meta[kMetaSel], blockIdx.x, gridDim.x);
@@ -183,18 +185,17 @@ __device__ __forceinline__ int4 block_sum4(int4 v, int4 *sh) {
 
 constexpr int kLayerBatch = 8;  // window layers whose statistics are loaded together
 
-// kMaxItems positions per thread at most (N <= kMaxItems * blockDim.x); instantiated for
-// 1, 2, 4 and 8 so that short canvases carry no unused per-item state.
+// Scores and commits canvas b with the whole CTA.  kMaxItems positions per thread at most
+// (N <= kMaxItems * blockDim.x); instantiated for 1, 2, 4 and 8 so that short canvases carry
+// no unused per-item state.  The merged row statistics are read through L2 (ld.cg): in the
+// fused merge-and-score kernel other CTAs of the same grid wrote them.
 template <int kMaxItems>
-__global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p) {
+__device__ __forceinline__ void score_canvas(const ScoreParams &p, const int b) {
     __shared__ ScanPair sh_scan[33];
     __shared__ int4 sh_sum[32];
     __shared__ int first_reject;
     __shared__ unsigned long long best_fb;
 
-    pdl_trigger();  // successors may launch now; they wait for this grid before reading
-    pdl_wait();
-    const int b = blockIdx.x;
     const int N = p.N;
     const int nmt = p.meta[kMetaMasked];
     const int K = p.K;
@@ -243,8 +244,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
                     const int k = k_hi - 1 - t;
                     if (k >= 0) {
                         const size_t rk = static_cast<size_t>(k) * nmt + q;
-                        a_b[t] = p.row_arg[rk];
-                        p_b[t] = p.row_pmax[rk];
+                        a_b[t] = __ldcg(p.row_arg + rk);
+                        p_b[t] = __ldcg(p.row_pmax + rk);
                     }
                 }
 #pragma unroll
@@ -278,7 +279,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
                     }
                 }
             }
-            H[j] = p.row_H[static_cast<size_t>(K - 1) * nmt + q];
+            H[j] = __ldcg(p.row_H + static_cast<size_t>(K - 1) * nmt + q);
             r = peak - conf[j];
             s = static_cast<float>(min(ki, p.k_max)) - p.w * r;
             high[j] = conf[j] >= tau;
@@ -389,11 +390,54 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p
     }
 }
 
+template <int kMaxItems>
+__global__ void __launch_bounds__(kScoreThreads, 1) k_score_commit(ScoreParams p) {
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
+    pdl_wait();
+    score_canvas<kMaxItems>(p, blockIdx.x);
+}
+
+// The step's last merge and the scoring of its single canvas in one grid: the CTAs merge
+// their rows; the one that finishes last (a device counter, zeroed by the compaction)
+// scores the canvas.  No CTA waits for another.  With no rows to merge, CTA 0 scores.
+template <int kMaxItems>
+__global__ void __launch_bounds__(kMergeThreads) k_merge_score(MergeArgs mg, int32_t *meta,
+                                                                const int32_t *sel_list,
+                                                                ScoreParams p) {
+    __shared__ int last;
+    pdl_trigger();
+    pdl_wait();
+    const int working = merge_pass_rows(mg, meta, sel_list, 0, meta[kMetaSel], blockIdx.x, gridDim.x);
+    if (working == 0) {
+        if (blockIdx.x != 0) return;
+    } else {
+        if (static_cast<int>(blockIdx.x) >= working) return;
+        __threadfence();  // this CTA's merged rows are visible before it is counted
+        __syncthreads();
+        if (threadIdx.x == 0) last = atomicAdd(&meta[kMetaMergeDone], 1) == working - 1;
+        __syncthreads();
+        if (!last) return;
+        __threadfence();
+    }
+    score_canvas<kMaxItems>(p, 0);
+}
+
 }  // namespace
 
 cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,
                          int grid, cudaStream_t s) {
-    return launch_pdl(k_merge, dim3(grid), dim3(256), 0, s, mg, meta, sel_list);
+    return launch_pdl(k_merge, dim3(grid), dim3(kMergeThreads), 0, s, mg, meta, sel_list);
+}
+
+cudaError_t launch_merge_score(const MergeArgs &mg, int32_t *meta, const int32_t *sel_list,
+                               int grid, const ScoreParams &p, cudaStream_t s) {
+    if (p.B != 1 || p.N > kFuseScoreMaxN) return cudaErrorInvalidValue;
+    const int items = (p.N + kMergeThreads - 1) / kMergeThreads;
+    const dim3 g(grid), t(kMergeThreads);
+    if (items <= 1) return launch_pdl(k_merge_score<1>, g, t, 0, s, mg, meta, sel_list, p);
+    if (items <= 2) return launch_pdl(k_merge_score<2>, g, t, 0, s, mg, meta, sel_list, p);
+    if (items <= 4) return launch_pdl(k_merge_score<4>, g, t, 0, s, mg, meta, sel_list, p);
+    return launch_pdl(k_merge_score<8>, g, t, 0, s, mg, meta, sel_list, p);
 }
 
 cudaError_t launch_band(const BandParams &p, cudaStream_t s) {

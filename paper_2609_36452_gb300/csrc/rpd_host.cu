@@ -270,10 +270,40 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         e = launch_compact(cp, c->stream);
     }
     if (e != cudaSuccess) return cuda_fail(e, "compaction launch");
+
+    // Scoring, scan and commit of every canvas (k_score_commit, or the last merge's grid).
+    ScoreParams sp{};
+    sp.mask = mask;
+    sp.q_of_pos = c->q_of_pos;
+    sp.canvas_off = c->canvas_off;
+    sp.meta = c->meta;
+    sp.row_arg = c->row_arg;
+    sp.row_pmax = c->row_pmax;
+    sp.row_H = c->row_H;
+    sp.out_commit = out_commit;
+    sp.out_token = out_token;
+    sp.out_stats = out_stats;
+    sp.dbg = c->dbg;
+    sp.B = B;
+    sp.N = N;
+    sp.K = c->K;
+    sp.theta_c = c->rule.theta_c;
+    sp.theta_s = c->rule.theta_s;
+    sp.w = c->rule.w;
+    sp.k_max = c->rule.k_max;
+    sp.window = c->rule.window;
+    sp.block = c->rule.block;
+    sp.lazy = lazy ? 1 : 0;
+    for (int b = 0; b < B; ++b) {
+        sp.tau[b] = tau[b];
+        sp.budget[b] = budget[b];
+    }
+    const bool fuse_score = B == 1 && N <= kFuseScoreMaxN;
+
     // One projection pass: gather + RMSNorm prologue, head statistics, merge.  Rows, layers
     // and positions of the pass come from the device-side meta words.
     const MergeArgs mg{c->partials, c->max_splits, c->row_arg, c->row_pmax, c->row_H};
-    auto pass = [&](const int32_t *sel_list) -> cudaError_t {
+    auto pass = [&](const int32_t *sel_list, bool last) -> cudaError_t {
         cudaError_t err;
         {
             KernelTimer t(c, 0);
@@ -298,9 +328,11 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         }
         if (err != cudaSuccess) return err;
         KernelTimer t(c, 2);
+        if (last && fuse_score)
+            return launch_merge_score(mg, c->meta, sel_list, c->num_sms * 4, sp, c->stream);
         return launch_merge(mg, c->meta, sel_list, c->num_sms * 4, c->stream);
     };
-    e = pass(nullptr);
+    e = pass(nullptr, !lazy);
     if (e == cudaSuccess && lazy) {
         {
             KernelTimer t(c, 2);
@@ -324,38 +356,15 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             for (int b = 0; b < B; ++b) bp.tau[b] = tau[b];
             e = launch_band(bp, c->stream);
         }
-        if (e == cudaSuccess) e = pass(c->sel_q);
+        if (e == cudaSuccess) e = pass(c->sel_q, true);
     }
     c->stall_next = false;
     if (e != cudaSuccess) return cuda_fail(e, "projection launch");
+    // The step's last merge also scores the canvas when there is a single canvas of at most
+    // kFuseScoreMaxN positions (one launch fewer); otherwise score/commit is its own launch.
+    if (fuse_score) return RPD_OK;
     {
         KernelTimer t(c, 3);
-        ScoreParams sp{};
-        sp.mask = mask;
-        sp.q_of_pos = c->q_of_pos;
-        sp.canvas_off = c->canvas_off;
-        sp.meta = c->meta;
-        sp.row_arg = c->row_arg;
-        sp.row_pmax = c->row_pmax;
-        sp.row_H = c->row_H;
-        sp.out_commit = out_commit;
-        sp.out_token = out_token;
-        sp.out_stats = out_stats;
-        sp.dbg = c->dbg;
-        sp.B = B;
-        sp.N = N;
-        sp.K = c->K;
-        sp.theta_c = c->rule.theta_c;
-        sp.theta_s = c->rule.theta_s;
-        sp.w = c->rule.w;
-        sp.k_max = c->rule.k_max;
-        sp.window = c->rule.window;
-        sp.block = c->rule.block;
-        sp.lazy = lazy ? 1 : 0;
-        for (int b = 0; b < B; ++b) {
-            sp.tau[b] = tau[b];
-            sp.budget[b] = budget[b];
-        }
         e = launch_score_commit(sp, c->stream);
     }
     if (e != cudaSuccess) return cuda_fail(e, "score/commit launch");

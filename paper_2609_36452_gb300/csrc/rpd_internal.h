@@ -46,6 +46,7 @@ enum MetaIndex : int {
     kMetaRowsTotal = 7,// rows projected by all passes of this step
     kMetaLazy = 8,     // 1 when this step projects lazily (two passes)
     kMetaUnitNext = 9, // next head work unit to claim (zeroed before each projection pass)
+    kMetaMergeDone = 10, // CTAs that finished the fused merge-and-score (zeroed per step)
     kMetaWords = 16
 };
 
@@ -194,5 +195,10 @@ cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t
                          int grid, cudaStream_t s);
 cudaError_t launch_band(const BandParams &p, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
+// The step's last merge fused with the scoring of its canvas (one canvas of at most
+// kFuseScoreMaxN positions); the separate score launch is then skipped.
+constexpr int kFuseScoreMaxN = 2048;
+cudaError_t launch_merge_score(const MergeArgs &mg, int32_t *meta, const int32_t *sel_list,
+                               int grid, const ScoreParams &p, cudaStream_t s);
 
 }  // namespace rpd

@@ -43,6 +43,7 @@ constexpr int kNaMaxRows = 1024;
 constexpr int kNaMaxD = 4096;
 constexpr int kNaMaxN = 1024;
 constexpr int kNaMaxSplits = 320;
+static_assert(kNaMaxN <= kFuseScoreMaxN, "the canvas is scored by the merge's last CTA");
 constexpr int kNaMaxDevices = 64;
 
 // Arena layout (byte offsets, each 256-byte aligned).
@@ -217,10 +218,8 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         if (e == cudaSuccess && pair_slots > 0)
             e = launch_head_stats_pair(tmU, tmW_pair, hp, dev->pair_grid, stream);
     }
-    if (e == cudaSuccess)
-        e = launch_merge(MergeArgs{partials, splits, row_arg, row_pmax, row_H}, meta, nullptr,
-                         dev->num_sms * 4, stream);
     if (e == cudaSuccess) {
+        // the merge's last CTA scores the canvas (N <= kNaMaxN <= kFuseScoreMaxN), as rpd_step does
         ScoreParams sp{};
         sp.mask = mask;
         sp.q_of_pos = q_of_pos;
@@ -243,7 +242,8 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         sp.block = rule.block;
         sp.tau[0] = tau;
         sp.budget[0] = budget;
-        e = launch_score_commit(sp, stream);
+        e = launch_merge_score(MergeArgs{partials, splits, row_arg, row_pmax, row_H}, meta, nullptr,
+                               dev->num_sms * 4, sp, stream);
     }
     if (e != cudaSuccess) {
         set_last_error((std::string("rpd_step_noalloc launch failed: ") + cudaGetErrorString(e)).c_str());

@@ -105,12 +105,13 @@ constexpr float kLn2 = 0.6931471805599453f;
 // and the entropy H = ln s - ln2 * t / s (Eq. 1) at layer * NMT + q.  Rows are handled by
 // groups of gs lanes, gs the smallest power of two keeping <= 8 partials per lane (at most
 // a warp), so that every lane's loads are issued together; this CTA's groups take row
-// slots first_group, first_group + group_stride, ... (in units of groups).
-__device__ void merge_pass_rows(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,
-                                int s_begin, int s_end, int cta_slot, int cta_slots) {
+// slots first_group, first_group + group_stride, ... (in units of groups).  Returns how many
+// of the cta_slots CTAs have rows to merge (the same value in every CTA).
+__device__ int merge_pass_rows(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,
+                               int s_begin, int s_end, int cta_slot, int cta_slots) {
     const int rows = meta[kMetaRows];
     const int sel = meta[kMetaSel];
-    if (rows <= 0 || sel <= 0 || s_end <= s_begin) return;
+    if (rows <= 0 || sel <= 0 || s_end <= s_begin) return 0;
     const int layers = rows / sel;
     const int layer0 = meta[kMetaLayer0];
     const int nmt = meta[kMetaMasked];
@@ -159,6 +160,7 @@ __device__ void merge_pass_rows(const MergeArgs &mg, const int32_t *meta, const 
             mg.row_H[out] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
         }
     }
+    return min(cta_slots, (total + groups - 1) / groups);
 }
 
 }  // namespace
