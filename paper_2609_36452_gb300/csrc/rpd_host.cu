@@ -104,9 +104,12 @@ struct rpd_ctx {
     CUtensorMap tmU{}, tmW{}, tmW_pair{};
     int pair_grid = 0;   // CTAs of the CTA-pair head kernel (2 x resident pairs; 0 = none)
 
-    // host-buffer entry point staging
+    // host-buffer entry point staging: device buffer, and a pinned host copy of its small
+    // part (mask, commit, tokens, stats) so that those move in one copy each way
     size_t stage_bytes = 0;
     uint8_t *stage = nullptr;
+    size_t stage_host_bytes = 0;
+    uint8_t *stage_host = nullptr;
 
     // profiling
     bool profile = false;
@@ -541,29 +544,37 @@ int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float ta
         if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(staging)");
         c->stage_bytes = need;
     }
+    const size_t small = need - off_mask;  // mask, commit, tokens, stats (with padding)
+    if (small > c->stage_host_bytes) {
+        if (c->stage_host) cudaFreeHost(c->stage_host);
+        c->stage_host = nullptr;
+        c->stage_host_bytes = 0;
+        cudaError_t e = cudaMallocHost(&c->stage_host, small);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMallocHost(staging)");
+        c->stage_host_bytes = small;
+    }
     uint8_t *d_hidden = c->stage;
     uint8_t *d_mask = c->stage + off_mask;
     uint8_t *d_commit = c->stage + off_commit;
     int32_t *d_token = reinterpret_cast<int32_t *>(c->stage + off_token);
     rpd_stats *d_stats = reinterpret_cast<rpd_stats *>(c->stage + off_stats);
+    uint8_t *h = c->stage_host;  // same layout as the device region from off_mask on
+    // tokens are written only where committed: the step starts from the caller's canvas
+    std::memcpy(h, mask, static_cast<size_t>(N));
+    std::memcpy(h + (off_token - off_mask), out_token, static_cast<size_t>(N) * 4);
     cudaError_t e = cudaMemcpyAsync(d_hidden, hidden, hid, cudaMemcpyHostToDevice, c->stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(d_mask, mask, N, cudaMemcpyHostToDevice, c->stream);
-    // tokens are written only where committed: start from the caller's canvas
     if (e == cudaSuccess)
-        e = cudaMemcpyAsync(d_token, out_token, static_cast<size_t>(N) * 4, cudaMemcpyHostToDevice,
-                            c->stream);
+        e = cudaMemcpyAsync(d_mask, h, off_stats - off_mask, cudaMemcpyHostToDevice, c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "host->device copy");
     int rc = run_step(c, d_hidden, d_mask, 1, N, &tau, &budget, d_commit, d_token, d_stats);
     if (rc) return rc;
-    e = cudaMemcpyAsync(mask, d_mask, N, cudaMemcpyDeviceToHost, c->stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(out_commit, d_commit, N, cudaMemcpyDeviceToHost, c->stream);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(out_token, d_token, static_cast<size_t>(N) * 4, cudaMemcpyDeviceToHost,
-                            c->stream);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(out_stats, d_stats, sizeof(rpd_stats), cudaMemcpyDeviceToHost, c->stream);
+    e = cudaMemcpyAsync(h, d_mask, small, cudaMemcpyDeviceToHost, c->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "device->host copy");
+    std::memcpy(mask, h, static_cast<size_t>(N));
+    std::memcpy(out_commit, h + (off_commit - off_mask), static_cast<size_t>(N));
+    std::memcpy(out_token, h + (off_token - off_mask), static_cast<size_t>(N) * 4);
+    std::memcpy(out_stats, h + (off_stats - off_mask), sizeof(rpd_stats));
     return RPD_OK;
 }
 
@@ -600,6 +611,7 @@ void rpd_destroy(rpd_ctx *c) {
     cudaStreamSynchronize(c->stream);
     c->free_scratch();
     if (c->stage) cudaFree(c->stage);
+    if (c->stage_host) cudaFreeHost(c->stage_host);
     for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
     delete c;
 }
