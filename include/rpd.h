@@ -114,7 +114,8 @@ int rpd_get_rule(const rpd_ctx *ctx, rpd_rule *rule);
 int rpd_set_stream(rpd_ctx *ctx, void *stream);
 
 /* Pre-size scratch for B canvases of N positions, so that later steps of that size
- * allocate nothing.  Steps grow scratch on demand otherwise (synchronising the device). */
+ * allocate nothing.  Steps grow scratch on demand otherwise (synchronising the device).
+ * Requires B >= 1 and N >= 1; B > 128 or N > 8192: RPD_ERR_UNSUPPORTED. */
 int rpd_reserve(rpd_ctx *ctx, int B, int N);
 
 /* How the window layers are projected (App. A.6, the layerwise projection).
@@ -191,6 +192,8 @@ int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int
 /* rpd_step with HOST buffers: copies hidden, mask and out_token in, runs the step, copies
  * mask, out_commit, out_token and out_stats back, and returns after the stream has finished.
  * mask and out_token are in/out: out_token (the canvas) changes only at committed positions.
+ * hidden is copied straight from the caller's buffer (pinned memory makes it faster); mask,
+ * out_token and the results travel through a pinned staging buffer, one copy each way.
  * Staging buffers are owned by the context (grown on demand; the first call of a larger size
  * allocates). */
 int rpd_step_host(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau,
