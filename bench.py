@@ -39,9 +39,9 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "333c34a81c872803"): 1.0505e9,     # profiles/k_head_stats_pair_llada_first_step.md
-    ("llada_tail_5_masked", "333c34a81c872803"): 1.0440e9,  # profiles/k_head_stats_llada_tail5.md
-    ("batched_serving", "333c34a81c872803"): 8.836e9,       # profiles/k_head_stats_pair_batched_serving.md
+    ("llada_first_step", "2bf1e6957f760dfb"): 1.0494e9,     # profiles/k_head_stats_pair_llada_first_step.md
+    ("llada_tail_5_masked", "2bf1e6957f760dfb"): 1.0437e9,  # profiles/k_head_stats_llada_tail5.md
+    ("batched_serving", "2bf1e6957f760dfb"): 8.822e9,       # profiles/k_head_stats_pair_batched_serving.md
 }
 
 
