@@ -122,6 +122,39 @@ def project_logits(h_bits, g_bits, W_bits, eps: float, v_chunk: int = 8192) -> n
     return z
 
 
+def project_logits_exact(h_bits, g_bits, W_bits, eps: float, v_chunk: int = 8192) -> np.ndarray:
+    """Reading D3, a diagnostic only: the same logits with no rounding anywhere,
+    z[r, v] = rho_r * sum_d g_d h_{r,d} W[v, d] in fp64 (the textbook RMSNorm followed by the
+    head).  Comparing it with ``project_logits`` measures what reading D1's single bf16
+    rounding of g*h changes."""
+    h_bits = np.ascontiguousarray(h_bits, dtype=np.uint16)
+    R, d = h_bits.shape
+    V = W_bits.shape[0]
+    rho = rms_factor(h_bits, eps)
+    x = bf16_to_f64(g_bits) * bf16_to_f64(h_bits)  # unrounded
+    z = np.empty((R, V), dtype=np.float64)
+    for v0 in range(0, V, v_chunk):
+        v1 = min(V, v0 + v_chunk)
+        z[:, v0:v1] = x @ bf16_to_f64(W_bits[v0:v1]).T
+    z *= rho[:, None]
+    return z
+
+
+def reading_gap(h_bits, g_bits, W_bits, eps: float) -> dict:
+    """Diagnostic: how far reading D1 lies from the unrounded reading D3 on the given rows -
+    the largest |p_D1(v) - p_D3(v)| over rows and tokens, the largest entropy difference, and
+    how many rows change their argmax."""
+    z1 = project_logits(h_bits, g_bits, W_bits, eps)
+    z3 = project_logits_exact(h_bits, g_bits, W_bits, eps)
+    p1, p3 = softmax(z1), softmax(z3)
+    return {
+        "rows": int(z1.shape[0]),
+        "max_abs_dp": float(np.max(np.abs(p1 - p3))),
+        "max_abs_dH": float(np.max(np.abs(entropy(p1) - entropy(p3)))),
+        "argmax_differs": int(np.sum(np.argmax(z1, axis=-1) != np.argmax(z3, axis=-1))),
+    }
+
+
 # ----------------------------------------------------------------------------------------
 # Readout of one predictive distribution (Eq. 1)
 # ----------------------------------------------------------------------------------------

@@ -73,6 +73,25 @@ def test_projection_equals_torch_rmsnorm_linear_when_gain_is_exact():
     np.testing.assert_allclose(z, ref, rtol=1e-12, atol=1e-12)
 
 
+def test_unrounded_reading_equals_torch_rmsnorm_linear():
+    """Reading D3 (diagnostic) is the textbook RMSNorm with a general gain followed by the
+    head: torch rms_norm + linear in fp64.  With power-of-two gains it equals reading D1."""
+    V, d, R = 89, 56, 6
+    W = _rand_head(V, d, 12)
+    gen = torch.Generator().manual_seed(13)
+    h = (torch.randn(R, d, generator=gen) * 3).to(torch.bfloat16)
+    gain = (1 + 0.1 * torch.randn(d, generator=gen)).to(torch.bfloat16)
+    eps = 1e-5
+    z3 = O.project_logits_exact(bf16_bits(h), bf16_bits(gain), bf16_bits(W), eps)
+    ref = F.linear(F.rms_norm(h.double(), (d,), gain.double(), eps), W.double()).numpy()
+    np.testing.assert_allclose(z3, ref, rtol=1e-12, atol=1e-12)
+    exact = torch.tensor([0.5, 1.0, 2.0, 4.0] * (d // 4), dtype=torch.bfloat16)
+    gap = O.reading_gap(bf16_bits(h), bf16_bits(exact), bf16_bits(W), eps)
+    assert gap["max_abs_dp"] == 0.0 and gap["argmax_differs"] == 0
+    gap = O.reading_gap(bf16_bits(h), bf16_bits(gain), bf16_bits(W), eps)
+    assert 0.0 < gap["max_abs_dp"] < 1e-2 and gap["rows"] == R
+
+
 def test_norm_operand_rounding_matches_torch():
     """For general gains the head operand is the bf16 RNE of g*h (torch's conversion)."""
     d, R = 64, 9
