@@ -250,6 +250,24 @@ def commit_sequential(masked, cand, H, beta: float) -> list:
     return A
 
 
+def accepted_prefix(masked, cand, H, beta: float) -> list:
+    """Closed form of the §3.2 rule, used only to cross-check ``commit_sequential`` at every
+    call: with Q_i the entropy of the masked non-candidates before i (a running sum in canvas
+    order), A_t is the candidates before the first candidate with Q_i > beta.  While every
+    earlier candidate was accepted E_i = Q_i term by term, and H >= 0 means that once one
+    candidate is rejected every later one is too; the sums are therefore bit-identical."""
+    A = []
+    q = 0.0
+    for i in range(len(masked)):
+        if cand[i]:
+            if q > beta:
+                break
+            A.append(i)
+        elif masked[i]:
+            q += float(H[i])
+    return A
+
+
 def fallback_commit(masked, c, window: int) -> int:
     """§3.2: when A_t is empty, commit the single prediction with the highest final
     confidence among the first ``window`` masked positions from the left (leftmost wins a
@@ -370,6 +388,7 @@ def rpd_step(hidden_bits, mask, g_bits, W_bits, eps: float, tau: float, budget: 
     masked = np.asarray(mask).astype(bool)
     sc = score_positions(hidden_bits, np.nonzero(masked)[0], g_bits, W_bits, eps, tau, rule)
     A = commit_sequential(masked, sc["cand"], sc["H"], budget)
+    assert A == accepted_prefix(masked, sc["cand"], sc["H"], budget)
     fb = -1
     if not A and masked.any():
         fb = fallback_commit(masked, sc["conf"], rule["window"])
@@ -442,6 +461,7 @@ def step_from_scores(masked, layer_argmax, layer_p_of_y, H, tau, budget, rule):
         conf[i] = layer_p_of_y[-1, i]
         cand[i] = is_candidate(conf[i], s_i, tau, rule["theta_c"], rule["theta_s"])
     A = commit_sequential(masked, cand, H, budget)
+    assert A == accepted_prefix(masked, cand, H, budget)
     fb = -1
     if not A and masked.any():
         fb = fallback_commit(masked, conf, rule["window"])

@@ -306,8 +306,9 @@ def test_sequential_equals_prefix_form_exhaustive():
                 cand[idx[np.array(cbits, dtype=bool)]] = True
                 H = rng.choice([0.0, 0.25, 0.5, 1.0, 3.0], size=n)
                 for beta in (0.0, 0.5, 1.0, 2.0, math.inf):
-                    assert O.commit_sequential(masked, cand, H, beta) == \
-                        _prefix_form(masked, cand, H, beta)
+                    seq = O.commit_sequential(masked, cand, H, beta)
+                    assert seq == _prefix_form(masked, cand, H, beta)
+                    assert seq == O.accepted_prefix(masked, cand, H, beta)
 
 
 def test_commit_set_is_unique_fixed_point_brute_force():
