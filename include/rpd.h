@@ -214,8 +214,9 @@ int rpd_kernel_times(rpd_ctx *ctx, double *ms /*[RPD_NUM_KERNELS]*/,
 /* rpd_step for callers that cannot allocate device memory.  (The paper has no counterpart:
  * this is a deployment variant of rpd_step.)  Some callers own every byte of device memory
  * themselves - a serving engine that plans one fixed arena, a plugin running inside another
- * framework's memory manager, code that must not allocate while its stream is captured - so
- * a library that calls cudaMalloc on their behalf is not an option.  This entry point takes
+ * framework's memory manager, a latency-critical loop in which a cudaMalloc (which can
+ * synchronise the device) is not acceptable - so a library that calls cudaMalloc on their
+ * behalf is not an option.  This entry point takes
  * no context and allocates nothing: it runs the same kernels as rpd_step with its scratch in
  * a static device array of this library (about 13 MiB, held on every GPU that loads the
  * library until the process exits).  The caller passes every input and output.

@@ -3,11 +3,11 @@
 // Who needs it: callers that are not allowed to allocate device memory themselves or to
 // let a library do it behind their back - for example a host application that plans all
 // of its device memory up front (a serving engine with a fixed arena, a plugin inside
-// another framework's memory manager), or code that must not call cudaMalloc while its
-// stream is being captured.  rpd_create/rpd_step allocate context scratch on demand; this
-// entry point instead runs the same kernels on a scratch arena that is a file-scope
-// __device__ array of this library, so it never calls cudaMalloc, cudaFree or any
-// allocating routine.  The caller still provides every input and output buffer.
+// another framework's memory manager), or a latency-critical loop in which a cudaMalloc,
+// which can synchronise the device, is not acceptable.  rpd_create/rpd_step allocate
+// context scratch on demand; this entry point instead runs the same kernels on a scratch
+// arena that is a file-scope __device__ array of this library, so it never calls
+// cudaMalloc, cudaFree or any allocating routine.  The caller still provides every input and output buffer.
 //
 // Limits of the arena (checked on every call, before any work is enqueued):
 //   K * N <= 1024 projected rows, d <= 4096, N <= 1024; the arena holds the compact head

@@ -1,8 +1,8 @@
 """rpd_step_noalloc: the entry point for callers that cannot allocate device memory.
 
 Such callers (a serving engine that owns one pre-planned arena, a plugin inside another
-framework's memory manager, code that may not allocate while its stream is captured)
-cannot let the library call cudaMalloc, so this entry point runs the step on a static
+framework's memory manager, a latency-critical loop where a device-synchronising cudaMalloc
+is not acceptable) cannot let the library call cudaMalloc, so this entry point runs the step on a static
 device array inside the library.  These tests call it through the C ABI and check that
 its outputs equal those of rpd_step (the context-based entry point) on the same inputs,
 for consecutive calls that leave different amounts of stale data in the shared array,
