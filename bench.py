@@ -601,7 +601,7 @@ def main():
     ap.add_argument("--tiling", choices=["auto", "single", "pair"], default="auto",
                     help="head contraction tiling (default: chosen per pass on the device)")
     ap.add_argument("--cpu-positions", type=int, default=32)
-    ap.add_argument("--ref-positions", type=int, default=8)
+    ap.add_argument("--ref-positions", type=int, default=32)
     ap.add_argument("--ref-seconds", type=float, default=150.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
