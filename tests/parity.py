@@ -259,11 +259,12 @@ def compare_rows(ref_rows: dict, got: dict, positions, K: int):
     return worst
 
 
-def compare_block_step(ref: O.StepResult, got: dict) -> ParityReport:
+def compare_block_step(ref: O.StepResult, got: dict, lazy: bool = False) -> ParityReport:
     """RPD-block: scores of the active block's positions, and the commit set against every
     outcome the oracle admits under its near-threshold decisions (same tolerances as
-    compare_step; no budget is involved)."""
+    compare_step; no budget is involved).  ``lazy`` as in compare_step."""
     rep = ParityReport()
+    band, edge = lazy_band(ref) if lazy else (np.ones_like(ref.masked), np.zeros_like(ref.masked))
     scored = np.isfinite(ref.conf)
     idx = np.nonzero(scored)[0]
     rep.n_masked = int(ref.masked.sum())
@@ -277,6 +278,8 @@ def compare_block_step(ref: O.StepResult, got: dict) -> ParityReport:
         assert rep.max_dconf < PROB_TOL and rep.max_dH < PROB_TOL
         for i in idx:
             for k in range(K):
+                if k < K - 1 and (not band[i] or edge[i]):
+                    continue  # lazy: not projected outside the band
                 if ref.layer_gap[k, i] >= DELTA:
                     assert got["layer_argmax"][k, i] == ref.layer_argmax[k, i], (k, i)
             if i not in free:

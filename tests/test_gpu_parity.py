@@ -464,6 +464,55 @@ def test_lazy_projection_llada_full(llada_head):
     print(rep, "band", n_band, lazy["stats"])
 
 
+@pytest.mark.parametrize("rule_name,block", [("llada", 0), ("dream", 0), ("llada", 32)])
+def test_lazy_projection_batched(rule_name, block):
+    """Lazy projection over several canvases with their own tau and budget (each canvas has
+    its own stability band), for both Table 4 profiles and for RPD-block: commits, tokens and
+    masks equal the all-layer step, every canvas matches its oracle step, and the rows
+    projected are each canvas's scored positions plus the earlier layers of its band."""
+    K, N, d, V, B = 4, 96, 256, 2048, 4
+    W, g = WL.make_head(V, d, 77, w_std=0.08)
+    hidden = torch.empty(K, B, N, d, dtype=torch.bfloat16)
+    masks = torch.empty(B, N, dtype=torch.uint8)
+    for b in range(B):
+        cv = WL.make_hidden(W, K, N, 7700 + b, WL.u_profile(N, 0.5, 3.0),
+                              WL.calibrated_sigma(V, d, 0.08, 3.0), flip_frac=0.15, a=torch.ones(K))
+        hidden[:, b] = cv.hidden
+        masks[b] = WL.uniform_fraction_mask(N, [1.0, 0.7, 0.4, 0.9][b], 7800 + b)
+    taus, budgets = [0.9, 0.8, 0.95, 0.7], [1.0, 3.0, 0.5, 2.0]
+    rule = dict(O.RULES[rule_name], theta_s=3.0, block=block)
+    outs = {}
+    for lazy in (False, True):
+        runner = DeviceRunner(W, g, K, rule=rule)
+        runner.ctx.set_projection(lazy)
+        try:
+            outs[lazy] = runner.step_batched(hidden, masks, taus, budgets)
+        finally:
+            runner.close()
+    rows_lazy = 0
+    for b in range(B):
+        eager, lazy = outs[False][b], outs[True][b]
+        assert np.array_equal(lazy["commit"], eager["commit"])
+        assert np.array_equal(lazy["new_mask"], eager["new_mask"])
+        sel = lazy["commit"] == 1
+        assert np.array_equal(lazy["token"][sel], eager["token"][sel])
+        if block:
+            ref = O.rpd_block_step(bits(hidden[:, b]), masks[b].numpy(), bits(g), bits(W), 1e-6,
+                                   taus[b], rule)
+            compare_block_step(ref, lazy, lazy=True)
+        else:
+            ref = O.rpd_step(bits(hidden[:, b]), masks[b].numpy(), bits(g), bits(W), 1e-6, taus[b],
+                             budgets[b], rule)
+            compare_step(ref, lazy, lazy=True)
+        scored = np.isfinite(ref.conf) & ref.masked
+        c = lazy["conf"]
+        band = scored & (c >= np.float32(rule["theta_c"])) & (c < np.float32(taus[b]))
+        rows_lazy += int(scored.sum()) + (K - 1) * int(band.sum())
+    # n_rows counts the rows of the whole call (all canvases)
+    assert outs[True][0]["stats"]["n_rows"] == rows_lazy
+    assert rows_lazy < outs[False][0]["stats"]["n_rows"]
+
+
 def test_auto_projection_picks_per_step(llada_head):
     """Automatic projection: lazy at the LLaDA first step (1024 rows: bound by the tensor
     cores), every layer when 5 positions remain (bound by streaming the head); commits equal
