@@ -1,6 +1,7 @@
 """rpd_step captured into a CUDA graph: with scratch reserved beforehand the step enqueues no
 allocation and no host synchronisation, so it can be captured once and replayed; replays
-give the same outputs as eager steps."""
+give the same outputs as eager steps, with one projection pass or two (lazy, or chosen on
+the device inside the replay)."""
 import numpy as np
 import pytest
 import torch
@@ -15,7 +16,8 @@ if not torch.cuda.is_available():  # collected on CPU machines, never run there
 import paper_2609_36452_gb300 as rpd  # noqa: E402
 
 
-def test_step_replays_from_cuda_graph():
+@pytest.mark.parametrize("projection", ["all", "lazy", "auto"])
+def test_step_replays_from_cuda_graph(projection):
     dev = torch.device("cuda:0")
     K, N, d, V = 4, 256, 1024, 8192
     W, g = WL.make_head(V, d, 21, w_std=0.08)
@@ -25,6 +27,7 @@ def test_step_replays_from_cuda_graph():
     ctx = rpd.Rpd(d, V, K)
     ctx.set_head(W, g)
     ctx.set_profile("llada")
+    ctx.set_projection(projection)
     ctx.reserve(1, N)
     mask0 = torch.ones(N, dtype=torch.uint8, device=dev)
 
