@@ -5,8 +5,9 @@
   compared score by score; the commitment of every canvas is checked by replaying the
   oracle's rule on the GPU's own scores (a property that holds at any size).
 * Decode trajectory at the LLaDA-8B head shape: at every step the invariants, the commit
-  rule replayed on the GPU's scores and two sampled positions against the oracle; the full
-  oracle at the first, a middle and the last step.
+  rule replayed on the GPU's scores, two sampled positions against the oracle, and the same
+  commits with the projection chosen per step on the device; the full oracle at the first,
+  a middle and the last step.
 """
 import math
 
@@ -90,13 +91,21 @@ def test_llada_trajectory(traj_head):
     gen = torch.Generator().manual_seed(4004)
     targets = torch.randint(0, V, (N,), generator=gen)
     runner = DeviceRunner(W, g, K, 1e-6, rule="llada")
+    auto = DeviceRunner(W, g, K, 1e-6, rule="llada")     # projection chosen per step
+    auto.ctx.set_projection("auto")
     mask = torch.ones(N, dtype=torch.uint8)
     checked = []
     steps = []
+    lazy_steps = 0
     try:
         for t in range(64):
             cv = WL.trajectory_hidden(W, K, N, seed=4, step=t, mask=mask, targets=targets)
             got = runner.step(cv.hidden, mask, 0.9, 1.0)
+            a = auto.step(cv.hidden, mask, 0.9, 1.0)
+            assert np.array_equal(a["commit"], got["commit"]) and np.array_equal(a["new_mask"], got["new_mask"])
+            sel = got["commit"] == 1
+            assert np.array_equal(a["token"][sel], got["token"][sel])
+            lazy_steps += a["stats"]["n_rows"] < got["stats"]["n_rows"]
             m = mask.numpy().astype(bool)
             st = got["stats"]
             assert st["status"] == 0 and st["n_masked"] == int(m.sum())
@@ -108,7 +117,9 @@ def test_llada_trajectory(traj_head):
                 break
     finally:
         runner.close()
+        auto.close()
     assert int(mask.sum()) <= 0.02 * N, "trajectory did not finish within 64 steps"
+    assert 0 < lazy_steps < len(steps), (lazy_steps, len(steps))   # both choices were taken
     # every step: the commit rule replayed on the GPU's own scores, and two sampled masked
     # positions projected by the oracle (one fp64 projection for all sampled rows)
     rule = O.RULES["llada"]
