@@ -617,6 +617,23 @@ def test_exact_argmax_tie_takes_lowest_token():
     assert np.all(got["token"][got["commit"] == 1] == lo)
 
 
+def test_all_zero_hidden_rows_give_uniform_predictions():
+    """A hidden row of zeros (eps > 0) normalises to zeros, so every logit is 0: the
+    prediction is uniform - c = 1/V, H = ln V, argmax the lowest token (index 0) on every
+    layer - and such positions are never candidates.  The other positions are unaffected."""
+    K, N, d, V = 3, 40, 256, 4100
+    case = small_case(71, K=K, N=N, d=d, V=V)
+    zero = [0, 7, 8, 39]
+    case["hidden"][:, zero] = 0
+    ref, got, rep = run_and_compare(case)
+    for i in zero:
+        assert np.all(got["layer_argmax"][:, i] == 0)
+        assert abs(got["conf"][i] - 1.0 / V) < 1e-7
+        assert abs(got["entropy"][i] - math.log(V)) < 2e-3
+        assert got["candidate"][i] == 0
+    print(rep)
+
+
 # ------------------------------------------------------------------ window and canvas limits
 
 @pytest.mark.parametrize("K,N,rule", [(16, 96, "llada"), (14, 96, "dream"), (64, 40, "llada")])
