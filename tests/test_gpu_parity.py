@@ -310,6 +310,19 @@ def test_invalid_arguments_on_gpu():
     with pytest.raises(rpd.RpdError) as e:
         ctx.set_rule(0.6, 3.5, 15.0, 0, 32)
     assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+    # TMA needs 16-byte aligned rows: a hidden tensor or head that starts 2 bytes off is
+    # refused before any work (outputs untouched)
+    flat = torch.zeros(3 * 8 * 256 + 1, dtype=torch.bfloat16, device=dev)
+    c.fill_(7)
+    with pytest.raises(rpd.RpdError) as e:
+        ctx.step(flat[1:].view(3, 8, 256), m, 0.9, 1.0, c, t, s)
+    assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+    torch.cuda.synchronize(dev)
+    assert torch.all(c == 7) and torch.all(m == 1)
+    Wflat = torch.zeros(4096 * 256 + 1, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(rpd.RpdError) as e:
+        ctx.set_head(Wflat[1:].view(4096, 256), g)
+    assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
     ctx.close()
 
 
