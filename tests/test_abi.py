@@ -70,3 +70,34 @@ def test_create_without_gpu_fails_cleanly(rpd):
     h = rpd.rpd_create(256, 4096, 3, ctypes.c_float(1e-6))
     assert not h
     assert rpd.rpd_last_error() != b""
+
+
+def test_header_is_plain_c_and_links(rpd, tmp_path):
+    """A C99 program that includes rpd.h, takes the address of every declared function and
+    calls the ones that need no GPU compiles with gcc and links against the library."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    names = declared_functions()
+    src = tmp_path / "use_rpd.c"
+    src.write_text(
+        "#include <stdio.h>\n#include \"rpd.h\"\n"
+        "typedef void (*any_fn)(void);\n"
+        "int main(void) {\n"
+        "  any_fn fns[] = {" + ", ".join(f"(any_fn){n}" for n in names) + "};\n"
+        "  rpd_rule r = {0.6f, 3.5f, 15.0f, 6, 32, 0};\n"
+        "  int rc = rpd_set_rule(NULL, &r);\n"
+        "  printf(\"%d %d %s\\n\", (int)(sizeof(fns) / sizeof(fns[0])), rc, rpd_version());\n"
+        "  return rc == RPD_ERR_INVALID_ARGUMENT ? 0 : 1;\n"
+        "}\n")
+    exe = tmp_path / "use_rpd"
+    libdir = os.path.dirname(rpd.lib_path)
+    r = subprocess.run([cc, "-std=c99", "-Wall", "-Werror", "-pedantic-errors", "-I",
+                        os.path.join(ROOT, "include"), str(src), "-o", str(exe), "-L", libdir,
+                        "-lrpd", f"-Wl,-rpath,{libdir}"], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    run = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert run.returncode == 0, run.stdout + run.stderr
+    assert run.stdout.split()[0] == str(len(names))
