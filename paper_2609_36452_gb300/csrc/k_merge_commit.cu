@@ -24,6 +24,10 @@
 //   first W masked positions (leftmost on ties, §3.2).  Then write the outputs, clear the
 //   committed mask bits and the per-canvas counters.  RPD-block skips the budget and takes
 //   the fallback over the active block.
+//
+// k_merge_score (grid; a single canvas of at most kFuseScoreMaxN positions): the step's last
+//   merge, after which the CTA that finishes last (a device counter) scores and commits the
+//   canvas exactly as k_score_commit does, saving a launch.
 #include "ptx.cuh"
 #include "rpd_internal.h"
 #include "step_common.cuh"
