@@ -20,7 +20,10 @@
  *  - Every int-returning function returns RPD_OK (0) or one of the RPD_ERR_* codes and
  *    records a message for rpd_last_error() (per host thread).  On an error return no
  *    output has been written unless the code is RPD_ERR_CUDA.
- *  - A context is not thread safe; use one context per host thread or serialise calls.
+ *  - A context is not thread safe; use one context per host thread or serialise calls.  A
+ *    context may be used from any host thread: each call that touches the GPU makes the
+ *    context's device (and its primary context) current for its duration and gives the
+ *    thread its previous device back.
  *  - Inputs must be finite; with eps = 0 an all-zero hidden row has no defined RMS factor.
  *    Sums of squares, logits and softmax statistics are fp32 (h^2 must not overflow fp32).
  */

@@ -45,17 +45,36 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    static const EncodeTiledFn fn = [] {  // initialised once, thread-safely
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
                                              cudaEnableDefault, &q) == cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
     return fn;
 }
+
+// Entry points that touch the GPU run with the context's device current and its primary
+// context bound to the calling thread - cudaSetDevice does both; a host thread that has not
+// used the CUDA runtime yet has no context, and the driver's tensor-map encoder then fails -
+// and give the thread its previous device back when they return.
+struct DeviceGuard {
+    int prev = -1;
+    cudaError_t err = cudaSuccess;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        err = cudaSetDevice(dev);
+    }
+    ~DeviceGuard() {
+        int now = -1;
+        if (prev >= 0 && cudaGetDevice(&now) == cudaSuccess && now != prev) cudaSetDevice(prev);
+    }
+    DeviceGuard(const DeviceGuard &) = delete;
+    DeviceGuard &operator=(const DeviceGuard &) = delete;
+};
 
 // Row-major bf16 matrix [rows][cols] -> 2-D tensor map with a (64 x box_rows) box and
 // 128-byte swizzling; out-of-range elements read as zero.
@@ -238,6 +257,8 @@ int check_call(const rpd_ctx *c, float tau, float budget) {
 int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const float *tau,
              const float *budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
     if (!c->W || !c->g) return fail(RPD_ERR_NO_HEAD, "rpd_set_head has not been called");
     if (B < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "B must be >= 1");
     if (B > kMaxBatch) return fail(RPD_ERR_UNSUPPORTED, "B must be <= %d", kMaxBatch);
@@ -407,6 +428,7 @@ rpd_ctx *rpd_create(int d, int V, int K, float eps) {
     c->K = K;
     c->eps = eps;
     cudaError_t e = cudaGetDevice(&c->device);
+    if (e == cudaSuccess) e = cudaSetDevice(c->device);  // binds the primary context to this thread
     if (e == cudaSuccess)
         e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
     if (e != cudaSuccess) {
@@ -431,6 +453,8 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
     if (!c || !W_head || !g_norm) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
     if (!aligned16(W_head) || !aligned16(g_norm))
         return fail(RPD_ERR_INVALID_ARGUMENT, "W_head and g_norm must be 16-byte aligned");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
     CUtensorMap m, m2;
     int rc = encode_bf16_2d(&m, W_head, static_cast<uint64_t>(c->V), c->d, kTileN);
     if (rc) return rc;
@@ -468,6 +492,8 @@ int rpd_reserve(rpd_ctx *c, int B, int N) {
     if (B < 1 || N < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "reserve: B and N must be >= 1");
     if (B > kMaxBatch || N > kMaxCanvas)
         return fail(RPD_ERR_UNSUPPORTED, "reserve: B <= %d, N <= %d", kMaxBatch, kMaxCanvas);
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
     return ensure_scratch(c, B, N);
 }
 
@@ -528,6 +554,8 @@ int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float ta
     if (N == 0) return run_step(c, nullptr, nullptr, 1, 0, &tau, &budget, nullptr, nullptr, nullptr);
     if (!hidden || !mask || !out_commit || !out_token || !out_stats)
         return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
     const size_t hid = static_cast<size_t>(c->K) * N * c->d * 2;
     const size_t off_mask = (hid + 255) & ~size_t(255);
     const size_t off_commit = off_mask + ((N + 255) & ~255);
@@ -586,6 +614,8 @@ int rpd_profile_enable(rpd_ctx *c, int enable) {
 
 int rpd_kernel_times(rpd_ctx *c, double *ms, int64_t *launches, int reset) {
     if (!c || !ms || !launches) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
     for (int k = 0; k < RPD_NUM_KERNELS; ++k) {
         ms[k] = 0.0;
         launches[k] = 0;
@@ -608,6 +638,7 @@ int rpd_kernel_times(rpd_ctx *c, double *ms, int64_t *launches, int reset) {
 
 void rpd_destroy(rpd_ctx *c) {
     if (!c) return;
+    DeviceGuard dg(c->device);
     cudaStreamSynchronize(c->stream);
     c->free_scratch();
     if (c->stage) cudaFree(c->stage);

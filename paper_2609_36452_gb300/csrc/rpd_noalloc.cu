@@ -85,16 +85,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
 
 bool encode_tile_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,
                      uint32_t box_rows) {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    static const EncodeTiledFn fn = [] {  // initialised once, thread-safely
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) != cudaSuccess ||
-            q != cudaDriverEntryPointSuccess)
-            return false;
-        fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
+    if (!fn) return false;
     cuuint64_t dims[2] = {cols, rows};
     cuuint64_t strides[1] = {cols * 2};
     cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
@@ -108,6 +108,8 @@ bool encode_tile_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t
 int setup_device(DeviceSetup **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return na_fail(RPD_ERR_CUDA, "cudaGetDevice failed");
+    // the same device; binds its primary context to a calling thread that has none yet
+    if (cudaSetDevice(dev) != cudaSuccess) return na_fail(RPD_ERR_CUDA, "cudaSetDevice failed");
     if (dev < 0 || dev >= kNaMaxDevices) return na_fail(RPD_ERR_UNSUPPORTED, "device index too large");
     std::lock_guard<std::mutex> lock(g_setup_mutex);
     DeviceSetup &s = g_setup[dev];

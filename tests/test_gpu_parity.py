@@ -630,6 +630,55 @@ def test_exact_argmax_tie_takes_lowest_token():
     assert np.all(got["token"][got["commit"] == 1] == lo)
 
 
+def test_two_contexts_on_two_host_threads():
+    """Two contexts, each driven by its own host thread on its own stream, step concurrently
+    (their kernels share the GPU); every step's outputs equal the same step run alone."""
+    import threading
+    import paper_2609_36452_gb300 as rpd
+    dev = torch.device("cuda:0")
+    cases = [small_case(91, K=4, N=256, d=1024, V=8192), small_case(92, K=3, N=200, d=512, V=6000)]
+
+    def run(case, stream, out, reps):
+        ctx = rpd.Rpd(case["d"], case["V"], case["K"])
+        try:
+            ctx.set_head(case["Wd"], case["gd"])
+            ctx.set_profile("llada")
+            ctx.set_stream(stream)
+            ctx.reserve(1, case["N"])
+            for _ in range(reps):
+                with torch.cuda.stream(stream):
+                    m = case["maskd"].clone()
+                    c = torch.zeros(case["N"], dtype=torch.uint8, device=dev)
+                    t = torch.full((case["N"],), -1, dtype=torch.int32, device=dev)
+                    s = torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev)
+                ctx.step(case["hd"], m, 0.9, 1.0, c, t, s)
+                stream.synchronize()
+                out.append((m.cpu(), c.cpu(), t.cpu(), s.cpu()))
+        finally:
+            ctx.close()
+
+    for case in cases:
+        case["Wd"], case["gd"] = case["W"].to(dev), case["g"].to(dev)
+        case["hd"], case["maskd"] = case["hidden"].to(dev), case["mask"].to(dev)
+    alone = []
+    for case in cases:
+        res = []
+        run(case, torch.cuda.Stream(dev), res, 1)
+        alone.append(res[0])
+    together = [[], []]
+    threads = [threading.Thread(target=run, args=(cases[i], torch.cuda.Stream(dev), together[i], 6))
+               for i in range(2)]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    for i in range(2):
+        assert len(together[i]) == 6
+        for res in together[i]:
+            for a, b in zip(res, alone[i]):
+                assert torch.equal(a, b)
+
+
 def test_all_zero_hidden_rows_give_uniform_predictions():
     """A hidden row of zeros (eps > 0) normalises to zeros, so every logit is 0: the
     prediction is uniform - c = 1/V, H = ln V, argmax the lowest token (index 0) on every
