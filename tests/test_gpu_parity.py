@@ -630,6 +630,49 @@ def test_exact_argmax_tie_takes_lowest_token():
     assert np.all(got["token"][got["commit"] == 1] == lo)
 
 
+def test_one_context_across_shapes_heads_and_rules():
+    """One context through a sequence a serving loop produces: a short canvas, a batch that
+    makes scratch grow, a short canvas again, a new head (same shape), and the Dream rule;
+    every step against its own oracle."""
+    K, d, V = 3, 256, 2048
+    case_a = small_case(501, K=K, N=50, d=d, V=V)
+    W2, g2 = WL.make_head(V, d, 502, w_std=0.08)
+    runner = DeviceRunner(case_a["W"], case_a["g"], K)
+    try:
+        got = runner.step(case_a["hidden"], case_a["mask"], 0.9, 1.0)
+        compare_step(oracle_step(case_a), got)
+        # batch of 3 canvases of 300: scratch grows
+        B, N = 3, 300
+        hidden = torch.empty(K, B, N, d, dtype=torch.bfloat16)
+        masks = torch.empty(B, N, dtype=torch.uint8)
+        for b in range(B):
+            cv = WL.make_hidden(case_a["W"], K, N, 510 + b, WL.u_profile(N, 0.5, 3.0),
+                                  WL.calibrated_sigma(V, d, 0.08, 3.0), flip_frac=0.1)
+            hidden[:, b] = cv.hidden
+            masks[b] = WL.uniform_fraction_mask(N, [1.0, 0.6, 0.3][b], 520 + b)
+        outs = runner.step_batched(hidden, masks, [0.9, 0.85, 0.9], [1.0, 2.0, 0.5])
+        for b in range(B):
+            ref = O.rpd_step(bits(hidden[:, b]), masks[b].numpy(), bits(case_a["g"]),
+                             bits(case_a["W"]), 1e-6, [0.9, 0.85, 0.9][b], [1.0, 2.0, 0.5][b], "llada")
+            compare_step(ref, outs[b])
+        # short canvas again on the grown scratch
+        got = runner.step(case_a["hidden"], case_a["mask"], 0.9, 1.0)
+        compare_step(oracle_step(case_a), got)
+        # a new head of the same shape, then the Dream rule
+        W2d, g2d = W2.to(runner.dev).contiguous(), g2.to(runner.dev).contiguous()
+        runner.ctx.set_head(W2d, g2d)
+        cv = WL.make_hidden(W2, K, 50, 530, WL.u_profile(50, 0.5, 3.0),
+                            WL.calibrated_sigma(V, d, 0.08, 3.0), flip_frac=0.1)
+        case_b = dict(case_a, W=W2, g=g2, hidden=cv.hidden)
+        got = runner.step(case_b["hidden"], case_b["mask"], 0.9, 1.0)
+        compare_step(oracle_step(case_b), got)
+        runner.set_rule("dream")
+        got = runner.step(case_b["hidden"], case_b["mask"], 0.85, 2.0)
+        compare_step(oracle_step(case_b, tau=0.85, budget=2.0, rule="dream"), got)
+    finally:
+        runner.close()
+
+
 def test_two_contexts_on_two_host_threads():
     """Two contexts, each driven by its own host thread on its own stream, step concurrently
     (their kernels share the GPU); every step's outputs equal the same step run alone."""
