@@ -148,6 +148,28 @@ def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
+def _arg(t, name: str, dtype: str, numel: int = None, cuda: bool = True):
+    """Refuse, before any GPU work, a tensor the C ABI would misread: on the wrong side
+    (host/device), of the wrong element type, not contiguous, or of the wrong size."""
+    if t is None or not hasattr(t, "data_ptr"):
+        raise RpdError(RPD_ERR_INVALID_ARGUMENT, f"{name}: a tensor is required")
+    if bool(t.is_cuda) != cuda:
+        raise RpdError(RPD_ERR_INVALID_ARGUMENT,
+                       f"{name}: must be a {'CUDA' if cuda else 'host (CPU)'} tensor")
+    if str(t.dtype) != "torch." + dtype:
+        raise RpdError(RPD_ERR_INVALID_ARGUMENT, f"{name}: dtype must be {dtype}, not {t.dtype}")
+    if not t.is_contiguous():
+        raise RpdError(RPD_ERR_INVALID_ARGUMENT, f"{name}: must be contiguous")
+    if numel is not None and t.numel() != numel:
+        raise RpdError(RPD_ERR_INVALID_ARGUMENT, f"{name}: {t.numel()} elements, expected {numel}")
+    return _ptr(t)
+
+
+_DEBUG_DTYPES = {"conf": "float32", "entropy": "float32", "persist": "int32", "drop": "float32",
+                 "stability": "float32", "candidate": "uint8", "layer_argmax": "int32",
+                 "layer_pmax": "float32"}
+
+
 class Rpd:
     """A context bound to torch tensors.  ``W`` ([V][d]) and ``g`` ([d]) are bf16 CUDA
     tensors that must outlive the context (the library borrows them)."""
@@ -172,9 +194,10 @@ class Rpd:
             pass
 
     def set_head(self, W, g):
-        assert W.is_cuda and g.is_cuda and W.is_contiguous() and g.is_contiguous()
+        pw = _arg(W, "W", "bfloat16", self.V * self.d)
+        pg = _arg(g, "g", "bfloat16", self.d)
         self._keep = [W, g]
-        _check(rpd_set_head(self.handle, _ptr(W), _ptr(g)))
+        _check(rpd_set_head(self.handle, pw, pg))
 
     def set_rule(self, theta_c, theta_s, w, k_max, window, block=0):
         _check(rpd_set_rule(self.handle,
@@ -223,7 +246,10 @@ class Rpd:
         if not tensors:
             _check(rpd_set_debug(self.handle, None))
             return
-        dbg = RpdDebug(*[_ptr(tensors.get(f)) if tensors.get(f) is not None else None
+        for f in tensors:
+            if f not in _DEBUG_DTYPES:
+                raise RpdError(RPD_ERR_INVALID_ARGUMENT, f"unknown debug output {f}")
+        dbg = RpdDebug(*[_arg(tensors[f], f, _DEBUG_DTYPES[f]) if tensors.get(f) is not None else None
                          for f, _ in RpdDebug._fields_])
         self._dbg_keep = tensors
         _check(rpd_set_debug(self.handle, ctypes.byref(dbg)))
@@ -232,27 +258,39 @@ class Rpd:
         """One canvas: hidden [K][N][d] bf16, mask [N] uint8 (in/out), out_commit [N] uint8,
         out_token [N] int32, out_stats int32 tensor of STATS_WORDS (an rpd_stats), all CUDA."""
         N = mask.numel()
-        _check(rpd_step(self.handle, _ptr(hidden), _ptr(mask), N, ctypes.c_float(tau),
-                        ctypes.c_float(budget), _ptr(out_commit), _ptr(out_token),
-                        _ptr(out_stats)))
+        args = (_arg(hidden, "hidden", "bfloat16", self.K * N * self.d), _arg(mask, "mask", "uint8"),
+                _arg(out_commit, "out_commit", "uint8", N), _arg(out_token, "out_token", "int32", N),
+                _arg(out_stats, "out_stats", "int32", STATS_WORDS))
+        _check(rpd_step(self.handle, args[0], args[1], N, ctypes.c_float(tau),
+                        ctypes.c_float(budget), *args[2:]))
 
     def step_batched(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
         """B canvases: hidden [K][B][N][d], mask/out_commit/out_token [B][N], out_stats
         [B][STATS_WORDS];
         tau and budget are length-B host sequences."""
         B, N = mask.shape
+        if len(tau) != B or len(budget) != B:
+            raise RpdError(RPD_ERR_INVALID_ARGUMENT, "tau and budget need one value per canvas")
+        args = (_arg(hidden, "hidden", "bfloat16", self.K * B * N * self.d),
+                _arg(mask, "mask", "uint8"), _arg(out_commit, "out_commit", "uint8", B * N),
+                _arg(out_token, "out_token", "int32", B * N),
+                _arg(out_stats, "out_stats", "int32", B * STATS_WORDS))
         ta = (ctypes.c_float * B)(*[float(x) for x in tau])
         bu = (ctypes.c_float * B)(*[float(x) for x in budget])
-        _check(rpd_step_batched(self.handle, _ptr(hidden), _ptr(mask), B, N,
+        _check(rpd_step_batched(self.handle, args[0], args[1], B, N,
                                 ctypes.cast(ta, ctypes.c_void_p), ctypes.cast(bu, ctypes.c_void_p),
-                                _ptr(out_commit), _ptr(out_token), _ptr(out_stats)))
+                                *args[2:]))
 
     def step_host(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
         """Host (CPU, ideally pinned) tensors; returns after the results are back."""
         N = mask.numel()
-        _check(rpd_step_host(self.handle, _ptr(hidden), _ptr(mask), N, ctypes.c_float(tau),
-                             ctypes.c_float(budget), _ptr(out_commit), _ptr(out_token),
-                             _ptr(out_stats)))
+        args = (_arg(hidden, "hidden", "bfloat16", self.K * N * self.d, cuda=False),
+                _arg(mask, "mask", "uint8", cuda=False),
+                _arg(out_commit, "out_commit", "uint8", N, cuda=False),
+                _arg(out_token, "out_token", "int32", N, cuda=False),
+                _arg(out_stats, "out_stats", "int32", STATS_WORDS, cuda=False))
+        _check(rpd_step_host(self.handle, args[0], args[1], N, ctypes.c_float(tau),
+                             ctypes.c_float(budget), *args[2:]))
 
     def profile(self, enable: bool):
         _check(rpd_profile_enable(self.handle, 1 if enable else 0))

@@ -101,3 +101,23 @@ def test_header_is_plain_c_and_links(rpd, tmp_path):
     run = subprocess.run([str(exe)], capture_output=True, text=True)
     assert run.returncode == 0, run.stdout + run.stderr
     assert run.stdout.split()[0] == str(len(names))
+
+
+def test_binding_refuses_tensors_the_abi_would_misread(rpd):
+    """The Python binding checks side (host/device), element type, contiguity and size of
+    every tensor before calling the C ABI, so a wrong tensor is an error, not a kernel
+    reading the wrong memory."""
+    import torch
+    ok = torch.zeros(6, dtype=torch.int32)
+    assert rpd._arg(ok, "x", "int32", 6, cuda=False) is not None
+    bad = [
+        (torch.zeros(6, dtype=torch.int32), dict(dtype="int32", numel=6, cuda=True)),     # host, not CUDA
+        (torch.zeros(6, dtype=torch.int64), dict(dtype="int32", numel=6, cuda=False)),    # element type
+        (torch.zeros(6, 2, dtype=torch.int32)[:, 0], dict(dtype="int32", numel=6, cuda=False)),  # strided
+        (torch.zeros(5, dtype=torch.int32), dict(dtype="int32", numel=6, cuda=False)),    # size
+        (None, dict(dtype="int32", numel=6, cuda=False)),
+    ]
+    for t, kw in bad:
+        with pytest.raises(rpd.RpdError) as e:
+            rpd._arg(t, "x", kw["dtype"], kw["numel"], cuda=kw["cuda"])
+        assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
