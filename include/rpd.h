@@ -105,7 +105,8 @@ rpd_ctx *rpd_create(int d, int V, int K, float eps);
 /* Borrow the LM head W_head ([V][d] bf16, row v = token v's output embedding, device,
  * 16-byte aligned) and the final-norm gain g_norm ([d] bf16, device, 16-byte aligned).
  * Both must stay valid until the context is destroyed or the head is replaced; the
- * library keeps no copy.  App. A.2: the model's own final normalisation and head. */
+ * library keeps no copy.  Host memory, or memory of another device, is refused with
+ * RPD_ERR_INVALID_ARGUMENT.  App. A.2: the model's own final normalisation and head. */
 int rpd_set_head(rpd_ctx *ctx, const void *W_head, const void *g_norm);
 
 /* Replace the rule parameters (Table 4).  Requires 0 <= theta_c, w >= 0, k_max >= 1,

@@ -455,6 +455,16 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
         return fail(RPD_ERR_INVALID_ARGUMENT, "W_head and g_norm must be 16-byte aligned");
     DeviceGuard dg(c->device);
     if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
+    // The head is read by TMA: it must be device memory of this context's device.
+    for (const void *p : {W_head, g_norm}) {
+        cudaPointerAttributes a{};
+        if (cudaPointerGetAttributes(&a, p) != cudaSuccess || a.device != c->device ||
+            (a.type != cudaMemoryTypeDevice && a.type != cudaMemoryTypeManaged)) {
+            cudaGetLastError();  // clear the (non-sticky) error the query may have recorded
+            return fail(RPD_ERR_INVALID_ARGUMENT,
+                        "W_head and g_norm must be device memory on the context's device");
+        }
+    }
     CUtensorMap m, m2;
     int rc = encode_bf16_2d(&m, W_head, static_cast<uint64_t>(c->V), c->d, kTileN);
     if (rc) return rc;

@@ -323,6 +323,12 @@ def test_invalid_arguments_on_gpu():
     with pytest.raises(rpd.RpdError) as e:
         ctx.set_head(Wflat[1:].view(4096, 256), g)
     assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+    # a host head handed to the C ABI directly (past the binding's own checks) is refused
+    import ctypes
+    W_host = torch.zeros(4096, 256, dtype=torch.bfloat16)
+    rc = rpd.rpd_set_head(ctx.handle, ctypes.c_void_p(W_host.data_ptr()), ctypes.c_void_p(g.data_ptr()))
+    assert rc == rpd.RPD_ERR_INVALID_ARGUMENT and b"device memory" in rpd.rpd_last_error()
+    ctx.set_head(W, g)  # still usable
     ctx.close()
 
 
