@@ -410,7 +410,9 @@ def run_rpd(args):
 
 
 def measure_e2e(ctx, case, args, world, barrier, reduce_max):
-    """Same step through rpd_step_host: pinned host inputs copied in, results read back."""
+    """Same step through rpd_step_host: inputs in pinned host memory (the step reads the masked
+    positions' hidden rows across the host link; mask and canvas are copied in), results read
+    back, every step inside the timed region."""
     N = case["N"]
     hid_h = case["hidden"].reshape(case["K"], N, case["d"]).contiguous().pin_memory()
     mask_h0 = case["mask"].reshape(N).clone()
@@ -428,10 +430,12 @@ def measure_e2e(ctx, case, args, world, barrier, reduce_max):
         mask_h.copy_(mask_h0)
         ctx.step_host(hid_h, mask_h, case["tau"], case["budget"], commit_h, token_h, stats_h)
     e2e_s = reduce_max(time.perf_counter() - t0)
-    h2d = hid_h.numel() * 2 + N + N * 4
-    d2h = N + N + N * 4 + 32
+    n_masked = int(mask_h0.sum())
+    h2d = case["K"] * n_masked * case["d"] * 2 + N + N * 4   # masked rows, mask, canvas tokens
+    d2h = N + N + N * 4 + 36                                  # mask, commits, tokens, stats
     return {"value": e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "api": "rpd_step_host (pinned host buffers)"}
+            "d2h_bytes_per_step": d2h,
+            "api": "rpd_step_host (pinned host buffers; hidden rows of masked positions read in place)"}
 
 
 def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st, world):

@@ -196,8 +196,10 @@ int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int
 /* rpd_step with HOST buffers: copies hidden, mask and out_token in, runs the step, copies
  * mask, out_commit, out_token and out_stats back, and returns after the stream has finished.
  * mask and out_token are in/out: out_token (the canvas) changes only at committed positions.
- * hidden is copied straight from the caller's buffer (pinned memory makes it faster); mask,
- * out_token and the results travel through a pinned staging buffer, one copy each way.
+ * hidden in pinned (page-locked) host memory is read in place by the step's gather kernel,
+ * so only the masked positions' rows cross the host link; hidden in other host memory is
+ * copied to the device first.  mask, out_token and the results travel through a pinned
+ * staging buffer, one copy each way.
  * Staging buffers are owned by the context (grown on demand; the first call of a larger size
  * allocates). */
 int rpd_step_host(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau,

@@ -566,7 +566,17 @@ int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float ta
         return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
     DeviceGuard dg(c->device);
     if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
-    const size_t hid = static_cast<size_t>(c->K) * N * c->d * 2;
+    // Pinned (page-locked, mapped) host memory is read in place by the gather kernel over the
+    // host link: only the masked positions' rows cross it, and no copy precedes the step.
+    // Any other host memory is copied to the device first.
+    const void *in_place = nullptr;
+    {
+        cudaPointerAttributes a{};
+        if (cudaPointerGetAttributes(&a, hidden) == cudaSuccess && a.type == cudaMemoryTypeHost)
+            in_place = a.devicePointer;
+        cudaGetLastError();  // clear the (non-sticky) error the query may have recorded
+    }
+    const size_t hid = in_place ? 0 : static_cast<size_t>(c->K) * N * c->d * 2;
     const size_t off_mask = (hid + 255) & ~size_t(255);
     const size_t off_commit = off_mask + ((N + 255) & ~255);
     const size_t off_token = off_commit + ((N + 255) & ~255);
@@ -591,7 +601,7 @@ int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float ta
         if (e != cudaSuccess) return cuda_fail(e, "cudaMallocHost(staging)");
         c->stage_host_bytes = small;
     }
-    uint8_t *d_hidden = c->stage;
+    const void *d_hidden = in_place ? in_place : c->stage;
     uint8_t *d_mask = c->stage + off_mask;
     uint8_t *d_commit = c->stage + off_commit;
     int32_t *d_token = reinterpret_cast<int32_t *>(c->stage + off_token);
@@ -600,7 +610,8 @@ int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float ta
     // tokens are written only where committed: the step starts from the caller's canvas
     std::memcpy(h, mask, static_cast<size_t>(N));
     std::memcpy(h + (off_token - off_mask), out_token, static_cast<size_t>(N) * 4);
-    cudaError_t e = cudaMemcpyAsync(d_hidden, hidden, hid, cudaMemcpyHostToDevice, c->stream);
+    cudaError_t e = cudaSuccess;
+    if (!in_place) e = cudaMemcpyAsync(c->stage, hidden, hid, cudaMemcpyHostToDevice, c->stream);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(d_mask, h, off_stats - off_mask, cudaMemcpyHostToDevice, c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "host->device copy");

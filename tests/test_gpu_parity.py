@@ -251,12 +251,16 @@ def test_largest_batch():
         assert (outs[b]["stats"]["n_committed"] >= 1) == (b % (N + 1) > 0)
 
 
-def test_host_entry_point_matches_device():
-    case = small_case(61, K=3, N=64)
+@pytest.mark.parametrize("pinned_hidden", [True, False])
+def test_host_entry_point_matches_device(pinned_hidden):
+    """rpd_step_host equals rpd_step: hidden in pinned memory is read in place, hidden in
+    pageable memory is copied to the device first."""
+    case = small_case(61, K=3, N=64, mask_frac=0.7)
     runner = DeviceRunner(case["W"], case["g"], 3)
     try:
         dev = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
-        hid = case["hidden"].contiguous().pin_memory()
+        hid = case["hidden"].contiguous()
+        hid = hid.pin_memory() if pinned_hidden else hid.clone()
         mask = case["mask"].clone().pin_memory()
         commit = torch.zeros(64, dtype=torch.uint8).pin_memory()
         token = torch.full((64,), -5, dtype=torch.int32).pin_memory()
