@@ -128,12 +128,16 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def make_workload(rank: int, masked: int = 0):
+def make_workload(rank: int, masked: int = 0, window: int = 0):
     """The LLaDA first-step canvas; ``masked`` > 0 keeps only the last ``masked`` positions
-    masked (the few-rows, head-streaming regime at the end of a decode trajectory)."""
+    masked (the few-rows, head-streaming regime at the end of a decode trajectory);
+    ``window`` > 0 projects that many final layers instead of 4 (16 is the paper's LLaDA
+    window, App. A.6)."""
     import workloads as WL
     W, g = WL.make_head(WL.LLADA_V, WL.LLADA_D, seed=2)
-    case = WL.llada_first_step(seed=2 + 97 * rank, W=W, g=g)
+    case = WL.llada_first_step(seed=2 + 97 * rank, W=W, g=g, K=window or 4)
+    if window:
+        case["name"] = f"llada_first_step_window{window}"
     if masked:
         m = torch.zeros(case["N"], dtype=torch.uint8)
         m[case["N"] - masked:] = 1
@@ -245,7 +249,7 @@ def load_workload(args, rank):
     """The benchmarked workload for this rank (each rank draws its own canvases)."""
     import workloads as WL
     if args.workload == "llada_first_step":
-        case = make_workload(rank, args.masked)
+        case = make_workload(rank, args.masked, args.window)
     elif args.workload == "dream_mid_decode":
         case = WL.dream_mid_decode(seed=3 + 97 * rank)
     elif args.workload == "batched_serving":
@@ -609,6 +613,9 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=150.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--window", type=int, default=0,
+                    help="LLaDA first step: project this many final layers (default 4; the "
+                         "paper's LLaDA window is 16)")
     ap.add_argument("--masked", type=int, default=0,
                     help="keep only the last N canvas positions masked (head-streaming regime)")
     args = ap.parse_args()

@@ -176,13 +176,14 @@ def tiny_step(seed: int = 1, calibrated: bool = False):
                 eps=1e-6, tau=0.9, budget=1.0, rule="llada", canvas=cv, seed=seed)
 
 
-def llada_first_step(seed: int = 2, kappa: float = DEFAULT_KAPPA, W=None, g=None):
-    """Batch 1, N=256 all masked, K=4, LLaDA-8B head (d=4096, V=126464), tau 0.9, budget 1.0.
+def llada_first_step(seed: int = 2, kappa: float = DEFAULT_KAPPA, W=None, g=None, K: int = 4):
+    """Batch 1, N=256 all masked, K=4 (or another window), LLaDA-8B head (d=4096, V=126464),
+    tau 0.9, budget 1.0.
 
     b_p is U-shaped from 0.3 (mid) to 4 (ends); 10% of positions flip their target in the
     penultimate window layer.
     """
-    K, N, d, V = 4, 256, LLADA_D, LLADA_V
+    N, d, V = 256, LLADA_D, LLADA_V
     if W is None:
         W, g = make_head(V, d, seed)
     b = u_profile(N, 0.3, 4.0)
