@@ -9,7 +9,6 @@
   commits with the projection chosen per step on the device; the full oracle at the first,
   a middle and the last step.
 """
-import math
 
 import numpy as np
 import pytest

@@ -2,7 +2,6 @@
 allocation and no host synchronisation, so it can be captured once and replayed; replays
 give the same outputs as eager steps, with one projection pass or two (lazy, or chosen on
 the device inside the replay)."""
-import numpy as np
 import pytest
 import torch
 

@@ -4,7 +4,6 @@ import math
 import os
 
 import numpy as np
-import torch
 
 from oracle import rpd_oracle as O
 from tests.test_oracle_pins import _tiny_inputs

@@ -11,7 +11,6 @@ and that sizes beyond the array's limits are refused before any work is done.
 The file is named so that pytest collects it last.
 """
 import ctypes
-import math
 
 import numpy as np
 import pytest
