@@ -251,12 +251,14 @@ def test_largest_batch():
         assert (outs[b]["stats"]["n_committed"] >= 1) == (b % (N + 1) > 0)
 
 
+@pytest.mark.parametrize("projection", ["all", "lazy"])
 @pytest.mark.parametrize("pinned_hidden", [True, False])
-def test_host_entry_point_matches_device(pinned_hidden):
-    """rpd_step_host equals rpd_step: hidden in pinned memory is read in place, hidden in
-    pageable memory is copied to the device first."""
-    case = small_case(61, K=3, N=64, mask_frac=0.7)
+def test_host_entry_point_matches_device(pinned_hidden, projection):
+    """rpd_step_host equals rpd_step: hidden in pinned memory is read in place (by both
+    projection passes when lazy), hidden in pageable memory is copied to the device first."""
+    case = small_case(61, K=3, N=64, mask_frac=0.7, a=torch.ones(3))
     runner = DeviceRunner(case["W"], case["g"], 3)
+    runner.ctx.set_projection(projection)
     try:
         dev = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
         hid = case["hidden"].contiguous()
