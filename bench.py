@@ -41,6 +41,7 @@ HEAD_TRAFFIC = {
     ("llada_first_step", "2bf1e6957f760dfb"): 1.0494e9,     # profiles/k_head_stats_pair_llada_first_step.md
     ("llada_tail_5_masked", "2bf1e6957f760dfb"): 1.0437e9,  # profiles/k_head_stats_llada_tail5.md
     ("batched_serving", "2bf1e6957f760dfb"): 8.822e9,       # profiles/k_head_stats_pair_batched_serving.md
+    ("dream_mid_decode", "2bf1e6957f760dfb"): 1.1033e9,     # profiles/k_head_stats_pair_dream_mid_decode.md
 }
 
 
