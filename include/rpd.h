@@ -166,8 +166,9 @@ int rpd_inject_stall(rpd_ctx *ctx);
 int rpd_set_debug(rpd_ctx *ctx, const rpd_debug *debug);
 
 /* One commit step for one canvas (§3).
- *   hidden     [K][N][d] bf16, device: pre-norm hidden state of each window layer at
- *              each canvas position (the final layer last).  Rows of unmasked
+ *   hidden     [K][N][d] bf16, device (or mapped page-locked host memory; anything else is
+ *              refused with RPD_ERR_INVALID_ARGUMENT): pre-norm hidden state of each window
+ *              layer at each canvas position (the final layer last).  Rows of unmasked
  *              positions are never read.
  *   mask       [N] uint8, device, in/out: 1 = masked.  Committed positions are set to 0.
  *   N          canvas length, 0 <= N <= 8192 (N = 0 is a no-op; N > 8192:
@@ -227,8 +228,12 @@ int rpd_kernel_times(rpd_ctx *ctx, double *ms /*[RPD_NUM_KERNELS]*/,
  * a static device array of this library (about 13 MiB, held on every GPU that loads the
  * library until the process exits).  The caller passes every input and output.
  *   W_head [V][d], g_norm [d], hidden [K][N][d]: bf16 device, 16-byte aligned;
- *   rule: NULL for the LLaDA profile of Table 4; mask/out_commit/out_token/out_stats and
- *   tau/budget as in rpd_step; stream: a cudaStream_t (NULL = legacy default stream).
+ *   rule: NULL for theta_c 0.6, theta_s 3.5, w 15, k_max 6, window 32, block 0 (the values
+ *   rpd_create installs); mask/out_commit/out_token/out_stats and tau/budget as in rpd_step,
+ *   with the same checks of the rule and thresholds; stream: a cudaStream_t (NULL = legacy
+ *   default stream).  W_head, g_norm and hidden that the current device cannot read (pageable
+ *   host memory, another device's memory) are refused with RPD_ERR_INVALID_ARGUMENT; hidden
+ *   may be mapped page-locked host memory.
  * Limits: K*N <= 1024, N <= 1024, d <= 4096 (plus rpd_create's shape rules); larger sizes
  * return RPD_ERR_UNSUPPORTED with a message naming the limit, before any work is enqueued.
  * All calls on a device share the one scratch array, which keeps the previous call's

@@ -93,8 +93,6 @@ int encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t rows, uint64_t c
     return RPD_OK;
 }
 
-bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-
 }  // namespace
 
 struct rpd_ctx {
@@ -233,24 +231,15 @@ struct KernelTimer {
 };
 
 int check_rule(const rpd_rule &r) {
-    if (!(r.theta_c >= 0.f) || !std::isfinite(r.theta_c))
-        return fail(RPD_ERR_INVALID_ARGUMENT, "theta_c must be finite and >= 0");
-    if (std::isnan(r.theta_s)) return fail(RPD_ERR_INVALID_ARGUMENT, "theta_s is NaN");
-    if (!(r.w >= 0.f) || !std::isfinite(r.w))
-        return fail(RPD_ERR_INVALID_ARGUMENT, "w must be finite and >= 0");
-    if (r.k_max < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "k_max must be >= 1");
-    if (r.window < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "window must be >= 1");
-    if (r.block < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "block must be >= 0");
-    return RPD_OK;
+    const char *msg = rule_error(r);
+    return msg ? fail(RPD_ERR_INVALID_ARGUMENT, "%s", msg) : RPD_OK;
 }
 
 int check_call(const rpd_ctx *c, float tau, float budget) {
-    if (!(tau > 0.f && tau <= 1.f)) return fail(RPD_ERR_INVALID_ARGUMENT, "tau must be in (0, 1]");
-    if (!(c->rule.theta_c < tau))
-        return fail(RPD_ERR_INVALID_ARGUMENT, "theta_c (%g) must be below tau (%g)",
-                    (double)c->rule.theta_c, (double)tau);
-    if (!(budget >= 0.f)) return fail(RPD_ERR_INVALID_ARGUMENT, "budget must be >= 0 (got %g)",
-                                      (double)budget);
+    const char *msg = call_error(c->rule, tau, budget);
+    if (msg)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "%s (theta_c %g, tau %g, budget %g)", msg,
+                    (double)c->rule.theta_c, (double)tau, (double)budget);
     return RPD_OK;
 }
 
@@ -273,6 +262,9 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
     if (!hidden || !mask || !out_commit || !out_token || !out_stats)
         return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
     if (!aligned16(hidden)) return fail(RPD_ERR_INVALID_ARGUMENT, "hidden must be 16-byte aligned");
+    if (!pointer_usable(hidden, c->device, true))
+        return fail(RPD_ERR_INVALID_ARGUMENT,
+                    "hidden must be device memory of the context's device or mapped page-locked host memory");
     int rc = ensure_scratch(c, B, N);
     if (rc) return rc;
 
@@ -456,15 +448,9 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
     DeviceGuard dg(c->device);
     if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
     // The head is read by TMA: it must be device memory of this context's device.
-    for (const void *p : {W_head, g_norm}) {
-        cudaPointerAttributes a{};
-        if (cudaPointerGetAttributes(&a, p) != cudaSuccess || a.device != c->device ||
-            (a.type != cudaMemoryTypeDevice && a.type != cudaMemoryTypeManaged)) {
-            cudaGetLastError();  // clear the (non-sticky) error the query may have recorded
-            return fail(RPD_ERR_INVALID_ARGUMENT,
-                        "W_head and g_norm must be device memory on the context's device");
-        }
-    }
+    if (!pointer_usable(W_head, c->device, false) || !pointer_usable(g_norm, c->device, false))
+        return fail(RPD_ERR_INVALID_ARGUMENT,
+                    "W_head and g_norm must be device memory on the context's device");
     CUtensorMap m, m2;
     int rc = encode_bf16_2d(&m, W_head, static_cast<uint64_t>(c->V), c->d, kTileN);
     if (rc) return rc;

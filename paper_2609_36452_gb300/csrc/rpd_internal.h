@@ -182,6 +182,46 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // Record the message returned by rpd_last_error() on this host thread.
 void set_last_error(const char *msg);
 
+// ------------------------------------------------------------------ argument checks
+// Shared by every entry point, so that they accept and refuse the same arguments.  Each
+// returns nullptr when the argument is acceptable, else the message to report.
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Rule parameters (Table 4): theta_c, w finite and >= 0, theta_s not NaN, k_max, window >= 1,
+// block >= 0.
+inline const char *rule_error(const rpd_rule &r) {
+    if (!(r.theta_c >= 0.f) || !(r.theta_c <= 3.402823466e38f)) return "theta_c must be finite and >= 0";
+    if (r.theta_s != r.theta_s) return "theta_s is NaN";
+    if (!(r.w >= 0.f) || !(r.w <= 3.402823466e38f)) return "w must be finite and >= 0";
+    if (r.k_max < 1) return "k_max must be >= 1";
+    if (r.window < 1) return "window must be >= 1";
+    if (r.block < 0) return "block must be >= 0";
+    return nullptr;
+}
+
+// Per-call thresholds: 0 < tau <= 1, theta_c < tau (Eq. 5 needs theta_c < theta_h), budget >= 0.
+inline const char *call_error(const rpd_rule &r, float tau, float budget) {
+    if (!(tau > 0.f && tau <= 1.f)) return "tau must be in (0, 1]";
+    if (!(r.theta_c < tau)) return "theta_c must be below tau";
+    if (!(budget >= 0.f)) return "budget must be >= 0";
+    return nullptr;
+}
+
+// Memory the kernels read with TMA (the head, the gain) must be device or managed memory of
+// `device`; memory the gather kernel reads with plain loads (hidden states) may also be
+// page-locked host memory mapped into the device's address space.  Any other pointer - pageable
+// host memory, another device's memory - would make the kernels fault, so it is refused.
+inline bool pointer_usable(const void *p, int device, bool host_mapped_ok) {
+    cudaPointerAttributes a{};
+    const bool ok = cudaPointerGetAttributes(&a, p) == cudaSuccess &&
+                    (((a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) &&
+                      a.device == device) ||
+                     (host_mapped_ok && a.type == cudaMemoryTypeHost && a.devicePointer == p));
+    cudaGetLastError();  // clear the (non-sticky) error the query may have recorded
+    return ok;
+}
+
 cudaError_t launch_compact(const CompactParams &p, cudaStream_t s);
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s);
 cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, const HeadParams &p,

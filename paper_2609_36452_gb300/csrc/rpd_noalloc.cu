@@ -16,9 +16,12 @@
 //   every GPU that loads this library until the process exits.
 //
 // Sharing: every call on a device uses the same arena and leaves its contents behind.
-// The step's status/count words are cleared at the start of each call; everything else
-// is fully rewritten before it is read.  Calls whose work overlaps on the GPU (two host
-// threads, or two streams) race on the arena: serialise them (one stream, or events).
+// The step's status/count words are cleared at the start of each call, and every array the
+// step reads is rewritten by the same call before it is read, with one exception: the last
+// head tile also reads the rows of the compact head operand past the call's live row count
+// (left over from an earlier call, or zero), and its epilogue discards what those rows
+// produce.  Calls whose work overlaps on the GPU (two host threads, or two streams) race on
+// the arena: serialise them (one stream, or events).
 //
 // Set-up: the first call on each device looks up the arena's device address with
 // cudaGetSymbolAddress (the array's name in host code is only a host-side stand-in, not a
@@ -65,6 +68,7 @@ static __device__ __align__(256) uint8_t g_noalloc_arena[kArenaBytes];
 
 struct DeviceSetup {
     bool ready = false;
+    int device = 0;
     uint8_t *arena = nullptr;  // device address of g_noalloc_arena on this device
     int num_sms = 0;
     int pair_grid = 0;         // CTAs of the CTA-pair head kernel (same choice as rpd_step)
@@ -124,6 +128,7 @@ int setup_device(DeviceSetup **out) {
         int sms = 0;
         e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         if (e != cudaSuccess) return na_fail(RPD_ERR_CUDA, "cudaDeviceGetAttribute failed");
+        s.device = dev;
         s.arena = static_cast<uint8_t *>(ptr);
         s.num_sms = sms;
         s.pair_grid = 2 * std::min(head_stats_pair_max_clusters(), sms / 2);
@@ -132,8 +137,6 @@ int setup_device(DeviceSetup **out) {
     *out = &s;
     return RPD_OK;
 }
-
-bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 }  // namespace
 
@@ -159,12 +162,8 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
         return na_fail(RPD_ERR_UNSUPPORTED, msg);
     }
     if (!(eps >= 0.f) || !std::isfinite(eps)) return na_fail(RPD_ERR_INVALID_ARGUMENT, "eps must be finite and >= 0");
-    if (!(rule.theta_c >= 0.f) || !(rule.w >= 0.f) || rule.k_max < 1 || rule.window < 1 ||
-        rule.block < 0 || std::isnan(rule.theta_s))
-        return na_fail(RPD_ERR_INVALID_ARGUMENT, "invalid rule");
-    if (!(tau > 0.f && tau <= 1.f) || !(rule.theta_c < tau))
-        return na_fail(RPD_ERR_INVALID_ARGUMENT, "tau must be in (0, 1] and above theta_c");
-    if (!(budget >= 0.f)) return na_fail(RPD_ERR_INVALID_ARGUMENT, "budget must be >= 0");
+    if (const char *m = rule_error(rule)) return na_fail(RPD_ERR_INVALID_ARGUMENT, m);
+    if (const char *m = call_error(rule, tau, budget)) return na_fail(RPD_ERR_INVALID_ARGUMENT, m);
     if (N == 0) return RPD_OK;
     if (!W_head || !g_norm || !hidden || !mask || !out_commit || !out_token || !out_stats)
         return na_fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
@@ -174,6 +173,14 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     DeviceSetup *dev = nullptr;
     int rc = setup_device(&dev);
     if (rc) return rc;
+    // The head and gain are read with TMA, the hidden states with plain loads: pointers the
+    // current device cannot read (pageable host memory, another device's memory) are refused
+    // here rather than becoming a fault in the kernels.
+    if (!pointer_usable(W_head, dev->device, false) || !pointer_usable(g_norm, dev->device, false))
+        return na_fail(RPD_ERR_INVALID_ARGUMENT, "W_head and g_norm must be device memory of the current device");
+    if (!pointer_usable(hidden, dev->device, true))
+        return na_fail(RPD_ERR_INVALID_ARGUMENT,
+                       "hidden must be device memory of the current device or mapped page-locked host memory");
     cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
     uint8_t *A = dev->arena;
     __nv_bfloat16 *u = reinterpret_cast<__nv_bfloat16 *>(A + kOffU);

@@ -91,16 +91,75 @@ def test_noalloc_matches_context_step_on_consecutive_calls():
         assert_same(run_context(case, tau, budget), run_noalloc(case, tau, budget))
 
 
-def test_noalloc_refuses_sizes_beyond_the_static_array():
-    case = make_case(83, K=5, N=256, d=256, V=4096, mask_frac=1.0)     # K*N = 1280 > 1024
+def call_noalloc(case, W, g, hidden, K=None, d=None, N=None, stream=None):
+    """One rpd_step_noalloc call with fresh, recognisable outputs; returns (rc, outputs)."""
+    N = case["N"] if N is None else N
     mask = case["mask"].clone()
     commit, token, stats = outputs(case["N"])
     p = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
-    rc = rpd.rpd_step_noalloc(p(case["W"]), p(case["g"]), case["d"], case["V"], case["K"],
-                              ctypes.c_float(1e-6), None, p(case["hidden"]), p(mask), case["N"],
-                              ctypes.c_float(0.9), ctypes.c_float(1.0), p(commit), p(token), p(stats),
-                              None)
-    assert rc == rpd.RPD_ERR_UNSUPPORTED
-    assert b"1024" in rpd.rpd_last_error()
+    rc = rpd.rpd_step_noalloc(p(W), p(g), case["d"] if d is None else d, case["V"],
+                              case["K"] if K is None else K, ctypes.c_float(1e-6), None, p(hidden),
+                              p(mask), N, ctypes.c_float(0.9), ctypes.c_float(1.0), p(commit),
+                              p(token), p(stats), stream)
     torch.cuda.synchronize(DEV)
-    assert torch.all(commit == 7) and torch.all(stats == -9) and torch.equal(mask, case["mask"])
+    return rc, (mask, commit, token, stats)
+
+
+def assert_untouched(case, outs):
+    mask, commit, token, stats = outs
+    assert torch.all(commit == 7) and torch.all(token == -5) and torch.all(stats == -9)
+    assert torch.equal(mask, case["mask"])
+
+
+@pytest.mark.parametrize("K,N,d,limit", [
+    (5, 256, 256, b"1024"),    # K*N = 1280 rows > 1024
+    (1, 1025, 256, b"1024"),   # N = 1025 > 1024
+    (1, 64, 4104, b"4096"),    # d = 4104 > 4096
+])
+def test_noalloc_refuses_sizes_beyond_the_static_array(K, N, d, limit):
+    case = make_case(83, K=K, N=N, d=d, V=4096, mask_frac=1.0)
+    rc, outs = call_noalloc(case, case["W"], case["g"], case["hidden"])
+    assert rc == rpd.RPD_ERR_UNSUPPORTED
+    assert limit in rpd.rpd_last_error()
+    assert_untouched(case, outs)
+
+
+def test_noalloc_refuses_memory_the_device_cannot_read():
+    """A head in ordinary (pageable) host memory would be a TMA source the GPU cannot read:
+    the call refuses it before any work is enqueued."""
+    case = make_case(84, K=2, N=64, d=256, V=4096, mask_frac=1.0)
+    W_host, g_host, h_host = case["W"].cpu(), case["g"].cpu(), case["hidden"].cpu()
+    for W, g, h in [(W_host, case["g"], case["hidden"]), (case["W"], g_host, case["hidden"]),
+                    (case["W"], case["g"], h_host)]:
+        rc, outs = call_noalloc(case, W, g, h)
+        assert rc == rpd.RPD_ERR_INVALID_ARGUMENT, rpd.rpd_last_error()
+        assert_untouched(case, outs)
+
+
+def test_noalloc_allocates_no_device_memory():
+    """After calls that have loaded every kernel the step uses, further calls with other
+    shapes leave the device's free memory unchanged (the scratch is the static array)."""
+    warm = [make_case(85, K=4, N=256, d=512, V=4096, mask_frac=1.0),
+            make_case(86, K=2, N=300, d=256, V=8192, mask_frac=0.7)]
+    fresh = [make_case(87, K=3, N=200, d=1024, V=5000, mask_frac=0.9),
+             make_case(88, K=1, N=400, d=768, V=4096, mask_frac=0.5)]
+    bufs = []
+    for case in warm + fresh:  # every output buffer exists before the measurement
+        bufs.append((case, outputs(case["N"]), case["mask"].clone()))
+    for case in warm:
+        rc, _ = call_noalloc(case, case["W"], case["g"], case["hidden"])
+        assert rc == rpd.RPD_OK, rpd.rpd_last_error()
+    torch.cuda.synchronize(DEV)
+    free0, _ = torch.cuda.mem_get_info(DEV)
+    p = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+    for case, (commit, token, stats), mask in bufs[len(warm):]:
+        rc = rpd.rpd_step_noalloc(p(case["W"]), p(case["g"]), case["d"], case["V"], case["K"],
+                                  ctypes.c_float(1e-6), None, p(case["hidden"]), p(mask), case["N"],
+                                  ctypes.c_float(0.9), ctypes.c_float(1.0), p(commit), p(token),
+                                  p(stats), None)
+        assert rc == rpd.RPD_OK, rpd.rpd_last_error()
+    torch.cuda.synchronize(DEV)
+    free1, _ = torch.cuda.mem_get_info(DEV)
+    assert free1 == free0, (free0, free1)
+    for case, (commit, token, stats), mask in bufs[len(warm):]:
+        assert int(stats[7]) == rpd.RPD_OK and int(stats[4]) >= 1
