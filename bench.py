@@ -251,14 +251,14 @@ def run_reference(args):
 
 def launches_per_step(case, args) -> int:
     """Kernels one rpd_step / rpd_step_batched call launches: the compaction; per projection
-    pass gather/norm, both head tilings (the one not chosen returns at once) and the merge;
-    the band selection before a second (lazy) pass; and score/commit, which the last merge
-    performs itself for a single canvas of at most 2048 positions."""
+    pass gather/norm, the head kernel and the merge; the band selection before a second (lazy)
+    pass; and score/commit, which the last merge performs itself for a single canvas of at
+    most 2048 positions."""
     B = case.get("B", 1)
     K, N = case["K"], case["N"]
     second_pass = args.projection == "lazy" or (args.projection == "auto" and K > 1 and K * B * N > 256)
     fused_score = B == 1 and N <= 2048
-    return 1 + 4 * (2 if second_pass else 1) + (1 if second_pass else 0) + (0 if fused_score else 1)
+    return 1 + 3 * (2 if second_pass else 1) + (1 if second_pass else 0) + (0 if fused_score else 1)
 
 
 def config_dict(case, R):
@@ -706,7 +706,7 @@ def main():
     ap.add_argument("--projection", choices=["all", "lazy", "auto"], default="all",
                     help="window layers projected: all (the step as defined), lazy (earlier "
                          "layers only for band positions), auto (chosen per step on the device)")
-    ap.add_argument("--tiling", choices=["auto", "single", "pair"], default="auto",
+    ap.add_argument("--tiling", choices=["auto", "pair", "rows_n"], default="auto",
                     help="head contraction tiling (default: chosen per pass on the device)")
     ap.add_argument("--cpu-positions", type=int, default=16,
                     help="positions of the oracle sample timed for cpu_baseline")

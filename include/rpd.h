@@ -141,15 +141,16 @@ int rpd_reserve(rpd_ctx *ctx, int B, int N);
 int rpd_set_projection(rpd_ctx *ctx, int mode);
 
 /* Tiling of the head contraction (no counterpart in the paper; it changes neither the
- * computed quantities nor, beyond fp32 summation order, their values).  By default
- * (RPD_TILING_AUTO) the step picks, on the device and per projection pass, the cheaper of:
- *   RPD_TILING_SINGLE  tiles of 128 rows x 256 vocabulary entries, one CTA each;
- *   RPD_TILING_PAIR    tiles of 256 rows x 256 entries on CTA pairs (tcgen05 cta_group::2).
- * Forcing one is for tests and measurements; RPD_TILING_PAIR on a device where no cluster
- * of two fits falls back to single-CTA tiles. */
+ * computed quantities nor, beyond fp32 summation order, their values).  Both tilings run on
+ * pairs of CTAs (tcgen05 cta_group::2).  By default (RPD_TILING_AUTO) the step picks, on the
+ * device and per projection pass, the cheaper of:
+ *   RPD_TILING_PAIR    tiles of 256 rows x 256 vocabulary entries (rows padded to 256);
+ *   RPD_TILING_ROWS_N  tiles of 256 vocabulary entries x a group of up to 512 rows, the rows
+ *                      on the MMA's N side (each group padded to a multiple of 32 rows).
+ * Forcing one is for tests and measurements. */
 #define RPD_TILING_AUTO 0
-#define RPD_TILING_SINGLE 1
-#define RPD_TILING_PAIR 2
+#define RPD_TILING_PAIR 1
+#define RPD_TILING_ROWS_N 2
 int rpd_set_head_tiling(rpd_ctx *ctx, int tiling);
 
 /* Diagnostics.  Every wait inside the step's kernels (mbarrier waits of the head kernels) is

@@ -66,9 +66,9 @@ RPD_PROJECT_LAZY = 1
 RPD_PROJECT_AUTO = 2
 PROJECTION_MODES = {"all": RPD_PROJECT_ALL, "lazy": RPD_PROJECT_LAZY, "auto": RPD_PROJECT_AUTO}
 RPD_TILING_AUTO = 0
-RPD_TILING_SINGLE = 1
-RPD_TILING_PAIR = 2
-HEAD_TILINGS = {"auto": RPD_TILING_AUTO, "single": RPD_TILING_SINGLE, "pair": RPD_TILING_PAIR}
+RPD_TILING_PAIR = 1
+RPD_TILING_ROWS_N = 2
+HEAD_TILINGS = {"auto": RPD_TILING_AUTO, "pair": RPD_TILING_PAIR, "rows_n": RPD_TILING_ROWS_N}
 
 
 class RpdError(RuntimeError):
@@ -226,15 +226,15 @@ class Rpd:
 
     def set_head_tiling(self, tiling):
         """Tiling of the head contraction: "auto" (default, chosen per pass on the device),
-        "single" (128-row tiles) or "pair" (256-row tiles on CTA pairs); for tests and
-        measurements."""
+        "pair" (256-row x 256-entry tiles on CTA pairs) or "rows_n" (256 entries x row groups
+        of up to 512 rows, padded to 32); for tests and measurements."""
         _check(rpd_set_head_tiling(self.handle, HEAD_TILINGS[tiling]))
 
     def set_wait_limit(self, microseconds: int):
         _check(rpd_set_wait_limit(self.handle, int(microseconds)))
 
     def inject_stall(self):
-        """Diagnostics: the next step's head kernels issue no loads; the step reports
+        """Diagnostics: the next step's head kernel issues no loads; the step reports
         RPD_ERR_TIMEOUT once its bounded waits run out."""
         _check(rpd_inject_stall(self.handle))
 

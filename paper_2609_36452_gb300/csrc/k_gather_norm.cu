@@ -87,25 +87,26 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
     __shared__ int lazy_on;
     const long long all_rows = static_cast<long long>(p.K) * carry;
     if (p.lazy == 2 && p.K > 1) {
-        int m_, s_;
+        int m_, s_, n_;
         const float e_all = choose_head_tiling(all_rows, p.num_n_tiles, p.max_splits,
-                                               p.single_slots, p.pair_slots, p.hbm_tiles, p.tiling, m_, s_);
-        const float e_fin = choose_head_tiling(carry, p.num_n_tiles, p.max_splits, p.single_slots,
-                                               p.pair_slots, p.hbm_tiles, p.tiling, m_, s_);
+                                               p.pair_slots, p.hbm_tiles, p.tiling, m_, s_, n_);
+        const float e_fin = choose_head_tiling(carry, p.num_n_tiles, p.max_splits,
+                                               p.pair_slots, p.hbm_tiles, p.tiling, m_, s_, n_);
         const long long guess = static_cast<long long>(kLazyBandGuess * (p.K - 1) * carry);
         const float e_band = choose_head_tiling(guess, p.num_n_tiles, p.max_splits,
-                                                p.single_slots, p.pair_slots, p.hbm_tiles, p.tiling, m_, s_);
+                                                p.pair_slots, p.hbm_tiles, p.tiling, m_, s_, n_);
         if (tid == 0) lazy_on = (e_fin + e_band < e_all) ? 1 : 0;
     } else if (tid == 0) {
         lazy_on = (p.lazy == 1 && p.K > 1) ? 1 : 0;
     }
     __syncthreads();
     const long long rows = lazy_on ? static_cast<long long>(carry) : all_rows;
-    int mode, splits;
-    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.single_slots, p.pair_slots,
-                       p.hbm_tiles, p.tiling, mode, splits);
+    int mode, splits, swap_rows;
+    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.pair_slots,
+                       p.hbm_tiles, p.tiling, mode, splits, swap_rows);
     if (tid == 0) {
         p.canvas_off[p.B] = carry;
+        p.meta[kMetaSwapRows] = swap_rows;
         p.meta[kMetaMasked] = carry;
         p.meta[kMetaRows] = static_cast<int>(rows);
         p.meta[kMetaStatus] = RPD_OK;

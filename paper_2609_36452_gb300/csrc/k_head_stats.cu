@@ -9,17 +9,20 @@
 // in TMEM) and reduced in the epilogue straight out of TMEM into per-row running
 // statistics in base-2 units (x = z * log2 e):
 //   m = max x,  s = sum 2^(x-m),  t = sum 2^(x-m) (x-m),  a = argmax (lowest index).
-// Logits never reach global memory.  Each work unit is (128-row tile, contiguous range of
+// Logits never reach global memory.  Each work unit is (row tile, contiguous range of
 // 256-wide vocabulary tiles); its statistics are written once per row as one partial
 // (float4) that the merge kernel combines.
 //
-// Persistent CTA, 6 warps:
-//   warp 0      TMA producer (one thread): u tile 128x64 and W tile 256x64 per stage
-//   warp 1      TMEM owner (alloc/dealloc 512 columns) and MMA issuer (one thread)
-//   warps 2..5  epilogue: warp w reads TMEM lanes 32*(w%4)..+31, one row per thread
-// Two 256-column fp32 accumulators (512 TMEM columns) let the epilogue of one tile run
-// under the MMAs of the next.  Every wait is bounded; a timeout latches RPD_ERR_TIMEOUT
-// in the step's status word and the CTA drains and exits.
+// One persistent kernel, launched as clusters of two CTAs (one per SM), serves two tilings;
+// the compaction kernel picks one per projection pass on the device and the kernel reads it
+// from the step's meta words.  Both run on CTA pairs (tcgen05 cta_group::2, M = 256):
+//   pair tiles:  256 rows (M, 128 per CTA) x 256 vocabulary entries (N);
+//   rows on N:   256 vocabulary entries (M, 128 per CTA) x a group of up to 512 rows (N,
+//                padded to a multiple of 32), so that a pass whose row count is not a multiple
+//                of 256 pads by at most 31 rows per group.
+// Roles: warp 0 TMA producer (one thread), warp 1 TMEM owner (512 columns) and MMA issuer
+// (one thread, even CTA), warps 2-5 (2-9 for rows on N) epilogue.  Every wait is bounded; a
+// timeout latches RPD_ERR_TIMEOUT in the step's status word and the CTA drains and exits.
 #include <atomic>
 
 #include "ptx.cuh"
@@ -78,17 +81,17 @@ struct UnitCursor {
     }
 };
 
-// Fold one 32-column chunk (already scaled to log2 units) into the running statistics.
+// Fold one 32-entry chunk of logits, column col0 + i in v[i], into the running statistics
+// (v is scaled to log2 units in place).
 template <bool kFull>
-__device__ __forceinline__ void fold_chunk(const float (&v)[32], float scale, int col0, int V,
+__device__ __forceinline__ void fold_chunk(float (&x)[32], float scale, int col0, int V,
                                            float &run_m, float &run_s, float &run_t,
                                            int &run_a) {
-    float x[32];
     float cmax = -INFINITY;
     int carg = 0;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
-        x[i] = v[i] * scale;
+        x[i] *= scale;
         if (!kFull && col0 + i >= V) x[i] = -INFINITY;
         if (x[i] > cmax) {
             cmax = x[i];
@@ -116,263 +119,96 @@ __device__ __forceinline__ void fold_chunk(const float (&v)[32], float scale, in
     }
 }
 
-__global__ void __launch_bounds__(kHeadThreads, 1)
-    k_head_stats(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW,
-                 HeadParams p) {
-    pdl_trigger();  // successors may launch now; they wait for this grid before reading
-    pdl_wait();     // row count, tiling, u and inv_rms come from the preceding kernels
-    if (p.meta[kMetaHeadMode] != 1 || p.meta[kMetaRows] == 0) return;  // pair tiling, or nothing to do
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t *sA = smem;
-    uint8_t *sB = smem + kStages * kStageBytesA;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kStages * (kStageBytesA + kStageBytesB));
-    uint64_t *full = bars;                  // [kStages] TMA -> MMA
-    uint64_t *empty = bars + kStages;       // [kStages] MMA -> TMA
-    uint64_t *acc_full = bars + 2 * kStages;      // [2] MMA -> epilogue
-    uint64_t *acc_empty = bars + 2 * kStages + 2; // [2] epilogue -> MMA
-    uint64_t *drain = bars + 2 * kStages + 4;     // [1] MMA completion at exit
-    uint64_t *unit_full = bars + 2 * kStages + 5; // [kUnitRing] producer -> MMA, epilogue
-    uint64_t *unit_empty = unit_full + kUnitRing; // [kUnitRing] MMA, epilogue -> producer
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(unit_empty + kUnitRing);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-    volatile int *unit_ring = abort_flag + 1;     // [kUnitRing] claimed unit indices
-
-    const int warp = threadIdx.x >> 5;
-    const int lane = threadIdx.x & 31;
-
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < kStages; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 1);
-        }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], 4);
-        }
-        for (int i = 0; i < kUnitRing; ++i) {
-            mbar_init(&unit_full[i], 1);
-            mbar_init(&unit_empty[i], 1 + 4);  // MMA issuer + 4 epilogue warps
-        }
-        mbar_init(drain, 1);
-        *abort_flag = 0;
-        fence_mbar_init();
-        tma_prefetch_desc(&tmU);
-        tma_prefetch_desc(&tmW);
-    }
-    if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
-    tc_fence_before_sync();
-    __syncthreads();
-    tc_fence_after_sync();
-    const uint32_t tmem_base = *tmem_slot;
-
-    const int rows = p.meta[kMetaRows];
-    TileWalk tw;
-    tw.init(rows, kTileM, p.V, p.d, p.meta[kMetaSplits]);
-    const int num_kb = (p.d + kTileK - 1) / kTileK;
-
-    if (warp == 0) {
-        if (lane == 0 && !p.stall) {
-            // ---------------------------------------------------------------- TMA producer
-            int stage = 0;
-            uint32_t phase = 0;
-            long long fills = 0;
-            bool ok = true;
-            UnitCursor uc;
-            while (ok) {
-                if (!mbar_wait_bounded(&unit_empty[uc.slot], uc.phase ^ 1u, abort_flag, p.wait_limit_ns))
-                    break;
-                const int claimed = atomicAdd(&p.meta[kMetaUnitNext], 1);
-                const int u = claimed < tw.units ? claimed : -1;
-                unit_ring[uc.slot] = u;
-                mbar_arrive(&unit_full[uc.slot]);
-                uc.advance();
-                if (u < 0) break;
-                int m, g, n0, n1;
-                tw.unit(u, m, g, n0, n1);
-                for (int n = n0; ok && n < n1; ++n) {
-                    for (int kb = 0; kb < num_kb; ++kb) {
-                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit_ns)) {
-                            ok = false;
-                            break;
-                        }
-                        mbar_arrive_expect_tx(&full[stage], kStageBytesA + kStageBytesB);
-                        tma_load_2d(sA + stage * kStageBytesA, &tmU, &full[stage], kb * kTileK,
-                                    m * kTileM);
-                        tma_load_2d(sB + stage * kStageBytesB, &tmW, &full[stage], kb * kTileK,
-                                    n * kTileN);
-                        ++fills;
-                        if (++stage == kStages) {
-                            stage = 0;
-                            phase ^= 1u;
-                        }
-                    }
-                }
-            }
-            // Drain: every issued copy must have landed before the CTA may exit (on the
-            // normal path they all have, since the MMA consumed them).
-            for (int s = 0; s < kStages; ++s) {
-                const long long n_s = fills / kStages + (s < fills % kStages ? 1 : 0);
-                if (n_s > 0) mbar_wait_drain(&full[s], static_cast<uint32_t>((n_s - 1) & 1), p.wait_limit_ns);
-            }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            // ---------------------------------------------------------------- MMA issuer
-            constexpr uint32_t idesc = idesc_bf16_f32(kTileM, kTileN);
-            int stage = 0;
-            uint32_t phase = 0;
-            uint32_t tile_iter = 0;
-            bool ok = true;
-            UnitCursor uc;
-            while (ok) {
-                if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns)) break;
-                const int u = unit_ring[uc.slot];
-                mbar_arrive(&unit_empty[uc.slot]);
-                uc.advance();
-                if (u < 0) break;
-                int m, g, n0, n1;
-                tw.unit(u, m, g, n0, n1);
-                for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
-                    const uint32_t acc = tile_iter & 1u;
-                    const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                    if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
-                                           p.wait_limit_ns)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after_sync();
-                    const uint32_t d_tmem = tmem_base + acc * kTileN;
-                    for (int kb = 0; kb < num_kb; ++kb) {
-                        if (!mbar_wait_bounded(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after_sync();
-                        const uint32_t a0 = smem_u32(sA + stage * kStageBytesA);
-                        const uint32_t b0 = smem_u32(sB + stage * kStageBytesB);
-#pragma unroll
-                        for (int kk = 0; kk < kTileK / 16; ++kk) {
-                            umma_bf16(d_tmem, smem_desc_sw128(a0 + kk * 32),
-                                      smem_desc_sw128(b0 + kk * 32), idesc,
-                                      (kb > 0 || kk > 0) ? 1u : 0u);
-                        }
-                        umma_commit(&empty[stage]);
-                        if (++stage == kStages) {
-                            stage = 0;
-                            phase ^= 1u;
-                        }
-                    }
-                    if (!ok) break;
-                    umma_commit(&acc_full[acc]);
-                }
-            }
-            // Drain: wait until every MMA this thread issued has completed.
-            umma_commit(drain);
-            mbar_wait_drain(drain, 0, p.wait_limit_ns);
-        }
-    } else {
-        // -------------------------------------------------------------------- epilogue
-        const int sub = warp & 3;  // TMEM sub-partition this warp may access
-        const int row_in_tile = sub * 32 + lane;
-        const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
-        uint32_t tile_iter = 0;
-        bool ok = true;
-        UnitCursor uc;
-        while (ok) {
-            if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns)) break;
-            const int u = unit_ring[uc.slot];
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&unit_empty[uc.slot]);
-            uc.advance();
-            if (u < 0) break;
-            int m, g, n0, n1;
-            tw.unit(u, m, g, n0, n1);
-            const int r = m * kTileM + row_in_tile;
-            const bool valid = r < rows;
-            const float scale = valid ? p.inv_rms[r] * kLog2e : 0.f;
-            float run_m = -INFINITY, run_s = 0.f, run_t = 0.f;
-            int run_a = 0;
-            for (int n = n0; n < n1; ++n, ++tile_iter) {
-                const uint32_t acc = tile_iter & 1u;
-                const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after_sync();
-                const int col_base = n * kTileN;
-                const bool full_tile = col_base + kTileN <= p.V;
-#pragma unroll 1
-                for (int c = 0; c < kTileN / 32; ++c) {
-                    float v[32];
-                    tmem_ld_32x32b_x32(lane_base + acc * kTileN + c * 32, v);
-                    if (full_tile)
-                        fold_chunk<true>(v, scale, col_base + c * 32, p.V, run_m, run_s, run_t, run_a);
-                    else
-                        fold_chunk<false>(v, scale, col_base + c * 32, p.V, run_m, run_s, run_t, run_a);
-                }
-                tc_fence_before_sync();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&acc_empty[acc]);
-            }
-            if (!ok) break;
-            if (valid) {
-                p.partials[static_cast<size_t>(r) * p.max_splits + g] =
-                    make_float4(run_m, run_s, run_t, __int_as_float(run_a));
-            }
-        }
-    }
-
-    __syncwarp();
-    tc_fence_before_sync();
-    __syncthreads();
-    tc_fence_after_sync();
-    if (*abort_flag && threadIdx.x == 0) atomicExch(&p.meta[kMetaStatus], RPD_ERR_TIMEOUT);
-    if (warp == 1) {
-        __syncwarp();
-        tmem_dealloc(tmem_base, kTmemCols);
-    }
+// Wait of a whole warp for a phase that takes long to complete (an accumulator): one lane polls,
+// the others wait at the warp barrier instead of competing for issue slots with the producer
+// and MMA threads, then every lane observes the completed phase itself (acquire).
+__device__ __forceinline__ bool warp_wait_bounded(uint64_t *bar, uint32_t parity,
+                                                  volatile int *abort, uint64_t limit_ns) {
+    int ok = 1;
+    if ((threadIdx.x & 31) == 0) ok = mbar_wait_bounded(bar, parity, abort, limit_ns) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (ok) mbar_try_wait(smem_u32(bar), parity);
+    return ok != 0;
 }
 
+// Combine two partial statistics (same rule as the merge kernel's): m = max, alpha =
+// 2^(m_j - m), s = sum alpha s_j, t = sum alpha (t_j + (m_j - m) s_j), argmax the lowest index
+// attaining m.
+__device__ __forceinline__ float4 merge_stat(float4 x, float4 y) {
+    if (y.y <= 0.f) return x;
+    if (x.y <= 0.f) return y;
+    const float m = fmaxf(x.x, y.x);
+    const float dx = x.x - m, dy = y.x - m;
+    const float ax = exp2f(dx), ay = exp2f(dy);
+    const int a = (x.x > y.x) ? __float_as_int(x.w)
+                : (y.x > x.x) ? __float_as_int(y.w) : min(__float_as_int(x.w), __float_as_int(y.w));
+    return make_float4(m, ax * x.y + ay * y.y, ax * fmaf(dx, x.y, x.z) + ay * fmaf(dy, y.y, y.z),
+                       __int_as_float(a));
+}
+
+// Shared memory of the head kernel: the operand ring, the rows-on-N transpose blocks, then the
+// barriers.
+struct HeadSmem {
+    uint8_t *ring;            // 1024-byte aligned
+    float *xpose;             // rows on N: [kSwapEpiWarps][32][33] transpose blocks, and at the
+                              // end of a unit the [4][kSwapMaxRows] statistics exchange
+    uint64_t *full;           // [kSwapMaxStages] TMA -> MMA (in the even CTA for pair tilings)
+    uint64_t *empty;          // [kSwapMaxStages] MMA -> TMA
+    uint64_t *acc_full;       // [2] MMA -> epilogue
+    uint64_t *acc_empty;      // [2] epilogue -> MMA (in the even CTA for pair tilings)
+    uint64_t *drain;          // [1] MMA completion at exit
+    uint64_t *unit_full;      // [kUnitRing] producer -> MMA, epilogue
+    uint64_t *unit_empty;     // [kUnitRing] MMA, epilogue -> producer
+    uint64_t *epi;            // [1] rows-on-N tiling: barrier of the epilogue warps
+    uint32_t *tmem_slot;
+    volatile int *abort_flag;
+    volatile int *unit_ring;  // [kUnitRing] claimed unit indices
+};
+
+__device__ __forceinline__ HeadSmem carve_smem(uint8_t *raw) {
+    HeadSmem s;
+    uint8_t *base = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    s.ring = base;
+    s.xpose = reinterpret_cast<float *>(base + kSwapStageBudget);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(base + kHeadRegionBytes);
+    s.full = bars;
+    s.empty = bars + kSwapMaxStages;
+    s.acc_full = bars + 2 * kSwapMaxStages;
+    s.acc_empty = s.acc_full + 2;
+    s.drain = s.acc_empty + 2;
+    s.unit_full = s.drain + 1;
+    s.unit_empty = s.unit_full + kUnitRing;
+    s.epi = s.unit_empty + kUnitRing;
+    s.tmem_slot = reinterpret_cast<uint32_t *>(s.epi + 1);
+    s.abort_flag = reinterpret_cast<volatile int *>(s.tmem_slot + 1);
+    s.unit_ring = s.abort_flag + 1;
+    return s;
+}
+
+static_assert((2 * kSwapMaxStages + 6 + 2 * kUnitRing) * 8 + 8 + 4 * kUnitRing <= kHeadBarrierBytes,
+              "barrier region");
 
 // ------------------------------------------------------------------------------------------
-// CTA-pair form (tcgen05 cta_group::2).  A pair (cluster of 2 CTAs) computes a tile of 256
-// rows x 256 vocabulary columns: CTA r of the pair stages rows [128r, 128r+128) of the row
+// Tiling 1: CTA pairs, rows on M (tcgen05 cta_group::2).  A pair (cluster of 2 CTAs) computes a tile of
+// 256 rows x 256 vocabulary columns: CTA r of the pair stages rows [128r, 128r+128) of the row
 // tile and W rows [128r, 128r+128) of the vocabulary tile; the even CTA issues
 // tcgen05.mma.cta_group::2 with M=256, N=256, which reads both CTAs' shared memory and
 // accumulates rows [128r, 128r+128) x all 256 columns into CTA r's TMEM.  Per SM and K-step
-// that is 32 KB of operands for the same MMA work the single-CTA tile does with 48 KB.
+// that is 32 KB of operands for the MMA work a single CTA's 128 x 256 tile would need 48 KB for.
 //
 // Barriers: full[s] lives in the even CTA and receives both CTAs' TMA completions (tx bytes
 // 64 KB per stage); empty[s], acc_full[a] and drain receive multicast commits from the MMA
 // thread in both CTAs; acc_empty[a] lives in the even CTA and counts the 4 epilogue warps
 // of both CTAs (8 arrivals).
-__global__ void __launch_bounds__(kHeadThreads, 1)
-    k_head_stats_pair(const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmW,
-                      HeadParams p) {
-    pdl_trigger();  // successors may launch now; they wait for this grid before reading
-    pdl_wait();     // row count, tiling, u and inv_rms come from the preceding kernels
-    if (p.meta[kMetaHeadMode] != 2 || p.meta[kMetaRows] == 0) return;  // single tiling, or nothing
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t *sA = smem;
-    uint8_t *sB = smem + kPairStages * kPairStageBytesA;
-    uint64_t *bars =
-        reinterpret_cast<uint64_t *>(smem + kPairStages * (kPairStageBytesA + kPairStageBytesB));
-    uint64_t *full = bars;                            // [kPairStages] (used in the even CTA)
-    uint64_t *empty = bars + kPairStages;             // [kPairStages]
-    uint64_t *acc_full = bars + 2 * kPairStages;      // [2]
-    uint64_t *acc_empty = bars + 2 * kPairStages + 2; // [2] (used in the even CTA)
-    uint64_t *drain = bars + 2 * kPairStages + 4;     // [1]
-    uint64_t *unit_full = bars + 2 * kPairStages + 5; // [kUnitRing] even producer -> all others
-    uint64_t *unit_empty = unit_full + kUnitRing;     // [kUnitRing] (used in the even CTA)
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(unit_empty + kUnitRing);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-    volatile int *unit_ring = abort_flag + 1;         // [kUnitRing] claimed unit indices
-
+__device__ __forceinline__ void head_pair(const CUtensorMap *tmU, const CUtensorMap *tmW,
+                                          const HeadParams &p, const HeadSmem &sm, int rows,
+                                          int splits) {
+    constexpr int kStageBytes = kPairStageBytesA + kPairStageBytesB;
+    uint64_t *full = sm.full, *empty = sm.empty, *acc_full = sm.acc_full,
+             *acc_empty = sm.acc_empty, *unit_full = sm.unit_full, *unit_empty = sm.unit_empty;
+    volatile int *abort_flag = sm.abort_flag;
+    volatile int *unit_ring = sm.unit_ring;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const uint32_t rank = cluster_ctarank();  // 0 = even CTA (issues the MMAs), 1 = odd
@@ -391,22 +227,21 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             // even CTA: its MMA issuer and 4 epilogue warps, the odd producer and 4 epilogue warps
             mbar_init(&unit_empty[i], 10);
         }
-        mbar_init(drain, 1);
+        mbar_init(sm.drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&tmU);
-        tma_prefetch_desc(&tmW);
+        tma_prefetch_desc(tmU);
+        tma_prefetch_desc(tmW);
     }
-    if (warp == 1) tmem_alloc_pair(tmem_slot, kTmemCols);
+    if (warp == 1) tmem_alloc_pair(sm.tmem_slot, kTmemCols);
     tc_fence_before_sync();
     __syncthreads();
     cluster_sync();  // both CTAs' barriers initialised before any cross-CTA signal
     tc_fence_after_sync();
-    const uint32_t tmem_base = *tmem_slot;
+    const uint32_t tmem_base = *sm.tmem_slot;
 
-    const int rows = p.meta[kMetaRows];
     TileWalk tw;
-    tw.init(rows, kPairTileM, p.V, p.d, p.meta[kMetaSplits]);
+    tw.init(rows, kPairTileM, p.V, p.d, splits);
     const int num_kb = (p.d + kTileK - 1) / kTileK;
 
     if (warp == 0) {
@@ -451,12 +286,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                             ok = false;
                             break;
                         }
-                        if (rank == 0)
-                            mbar_arrive_expect_tx(&full[stage], 2 * (kPairStageBytesA + kPairStageBytesB));
+                        if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes);
                         const uint32_t fb = full0 + static_cast<uint32_t>(stage * sizeof(uint64_t));
-                        tma_load_2d_pair(sA + stage * kPairStageBytesA, &tmU, fb, kb * kTileK,
+                        uint8_t *st = sm.ring + stage * kStageBytes;
+                        tma_load_2d_pair(st, tmU, fb, kb * kTileK,
                                          m * kPairTileM + static_cast<int>(rank) * kPairHalfRows);
-                        tma_load_2d_pair(sB + stage * kPairStageBytesB, &tmW, fb, kb * kTileK,
+                        tma_load_2d_pair(st + kPairStageBytesA, tmW, fb, kb * kTileK,
                                          n * kTileN + static_cast<int>(rank) * kPairHalfRows);
                         ++fills;
                         if (++stage == kPairStages) {
@@ -509,8 +344,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                                 break;
                             }
                             tc_fence_after_sync();
-                            const uint32_t a0 = smem_u32(sA + stage * kPairStageBytesA);
-                            const uint32_t b0 = smem_u32(sB + stage * kPairStageBytesB);
+                            const uint32_t a0 = smem_u32(sm.ring + stage * kStageBytes);
+                            const uint32_t b0 = a0 + kPairStageBytesA;
 #pragma unroll
                             for (int kk = 0; kk < kTileK / 16; ++kk) {
                                 umma_bf16_pair(d_tmem, smem_desc_sw128(a0 + kk * 32),
@@ -527,12 +362,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                         umma_commit_pair_multicast(&acc_full[acc], 0x3);
                     }
                 }
-                umma_commit_pair_multicast(drain, 0x3);
+                umma_commit_pair_multicast(sm.drain, 0x3);
             }
             // Both CTAs: every MMA writing this CTA's TMEM has completed before it is freed.
-            mbar_wait_drain(drain, 0, p.wait_limit_ns);
+            mbar_wait_drain(sm.drain, 0, p.wait_limit_ns);
         }
-    } else {
+    } else if (warp < 6) {
         // ---------------------------------------------------------- epilogue (both CTAs)
         const int sub = warp & 3;
         const int row_in_tile = static_cast<int>(rank) * kPairHalfRows + sub * 32 + lane;
@@ -561,7 +396,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             for (int n = n0; n < n1; ++n, ++tile_iter) {
                 const uint32_t acc = tile_iter & 1u;
                 const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
+                if (!warp_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
                     ok = false;
                     break;
                 }
@@ -601,12 +436,356 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     }
 }
 
+// Barrier of the rows-on-N epilogue's 256 threads: every thread arrives (release) and waits
+// for the phase (acquire), bounded like every other wait.  Returns false if it gave up.
+__device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, volatile int *abort,
+                                         uint64_t limit_ns) {
+    mbar_arrive(bar);
+    const bool ok = mbar_wait_bounded(bar, phase, abort, limit_ns);
+    phase ^= 1u;
+    return ok;
+}
+
+// ------------------------------------------------------------------------------------------
+// Tiling 2: "rows on N" CTA pairs.  The pair's MMA (cta_group::2, M = 256) takes the head as
+// its A operand - CTA r stages vocabulary rows [256n + 128r, +128) of tile n, 16 KB per
+// K-step - and a group of G_r rows of u as its B operand (N = G_r, a multiple of 32 up to
+// 512): the first N/2 columns come from the even CTA's shared memory, the rest from the odd
+// CTA's.  A group of more than 256 rows is issued as two MMAs (N = 256 and N = G_r - 256,
+// TMEM columns [0, 256) and [256, G_r)); a group of at most 256 rows is double-buffered in
+// TMEM.  So CTA r's TMEM holds logits for 128 vocabulary entries (lanes) x the group's rows
+// (columns): per row the softmax statistics reduce across lanes.  The epilogue (8 warps; the
+// two warps that share a TMEM sub-partition take alternate 32-column chunks) loads a 32 x 32
+// block, transposes it through shared memory so that each thread holds one row's 32
+// vocabulary entries, and folds them into that row's running statistics.  At the end of a
+// work unit the four sub-partitions' statistics of each row are combined through shared
+// memory and each CTA writes one partial per row (the merge sees 2 partials per split).
+// Each MMA's share of u in a stage is one TMA copy, from the tensor map whose box has that
+// share's height (16 to 128 rows).
+__device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps] */,
+                                          const CUtensorMap *tmW,
+                                          const HeadParams &p, const HeadSmem &sm, int rows,
+                                          int splits, int ng) {
+    uint64_t *full = sm.full, *empty = sm.empty, *acc_full = sm.acc_full,
+             *acc_empty = sm.acc_empty, *unit_full = sm.unit_full, *unit_empty = sm.unit_empty;
+    volatile int *abort_flag = sm.abort_flag;
+    volatile int *unit_ring = sm.unit_ring;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    // group geometry: columns of the two MMAs, accumulator buffers, ring depth
+    const int n0 = ng < kPairTileM ? ng : kPairTileM;
+    const int n1 = ng - n0;
+    const int nbuf = ng <= kPairTileM ? 2 : 1;
+    const int stage_b = (ng / 2) * kTileK * 2;
+    const int stage_bytes = kSwapStageBytesA + stage_b;
+    int stages = kSwapStageBudget / stage_bytes;
+    stages = stages < kSwapMaxStages ? stages : kSwapMaxStages;
+    constexpr int kEpiThreads = 32 * kSwapEpiWarps;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < stages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_empty[i], 2 * kSwapEpiWarps);
+        }
+        for (int i = 0; i < kUnitRing; ++i) {
+            mbar_init(&unit_full[i], 1);
+            // even CTA: its MMA issuer and epilogue warps; odd CTA: its producer and epilogue warps
+            mbar_init(&unit_empty[i], 2 + 2 * kSwapEpiWarps);
+        }
+        mbar_init(sm.epi, kEpiThreads);
+        mbar_init(sm.drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tma_prefetch_desc(&tmUrows[(n0 / 2) / kUBoxRows - 1]);
+        if (n1 > 0) tma_prefetch_desc(&tmUrows[(n1 / 2) / kUBoxRows - 1]);
+        tma_prefetch_desc(tmW);
+    }
+    if (warp == 1) tmem_alloc_pair(sm.tmem_slot, kTmemCols);
+    tc_fence_before_sync();
+    __syncthreads();
+    cluster_sync();
+    tc_fence_after_sync();
+    const uint32_t tmem_base = *sm.tmem_slot;
+
+    TileWalk tw;
+    tw.init(rows, ng, p.V, p.d, splits);
+    const int num_kb = (p.d + kTileK - 1) / kTileK;
+
+    if (warp == 0) {
+        if (lane == 0 && !p.stall) {
+            // ------------------------------------------------------- TMA producer (both CTAs)
+            const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);
+            const uint32_t unit_full1 = mapa_shared(smem_u32(&unit_full[0]), 1);
+            const uint32_t unit_ring1 = mapa_shared(smem_u32(const_cast<int *>(&unit_ring[0])), 1);
+            const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
+            const int half0 = n0 / 2, half1 = n1 / 2;  // rows this CTA stages for each MMA
+            // one copy per MMA's share of u: the map whose box is that many rows high
+            const CUtensorMap *map0 = &tmUrows[half0 / kUBoxRows - 1];
+            const CUtensorMap *map1 = &tmUrows[(half1 > 0 ? half1 : kUBoxRows) / kUBoxRows - 1];
+            int stage = 0;
+            uint32_t phase = 0;
+            long long fills = 0;
+            bool ok = true;
+            UnitCursor uc;
+            while (ok) {
+                int u;
+                if (rank == 0) {
+                    if (!mbar_wait_bounded_cluster(&unit_empty[uc.slot], uc.phase ^ 1u, abort_flag,
+                                                   p.wait_limit_ns))
+                        break;
+                    const int claimed = atomicAdd(&p.meta[kMetaUnitNext], 1);
+                    u = claimed < tw.units ? claimed : -1;
+                    unit_ring[uc.slot] = u;
+                    st_shared_cluster(unit_ring1 + static_cast<uint32_t>(uc.slot * sizeof(int)), u);
+                    mbar_arrive(&unit_full[uc.slot]);
+                    mbar_arrive_cluster(unit_full1 + static_cast<uint32_t>(uc.slot * sizeof(uint64_t)));
+                } else {
+                    if (!mbar_wait_bounded_cluster(&unit_full[uc.slot], uc.phase, abort_flag,
+                                                   p.wait_limit_ns))
+                        break;
+                    u = unit_ring[uc.slot];
+                    mbar_arrive_cluster(unit_empty0 + static_cast<uint32_t>(uc.slot * sizeof(uint64_t)));
+                }
+                uc.advance();
+                if (u < 0) break;
+                int m, g, v0, v1;
+                tw.unit(u, m, g, v0, v1);
+                const int rows0 = m * ng + static_cast<int>(rank) * half0;
+                const int rows1 = m * ng + kPairTileM + static_cast<int>(rank) * half1;
+                const int w_off = static_cast<int>(rank) * kPairHalfRows;
+                for (int n = v0; ok && n < v1; ++n) {
+                    for (int kb = 0; kb < num_kb; ++kb) {
+                        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit_ns)) {
+                            ok = false;
+                            break;
+                        }
+                        if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * stage_bytes);
+                        const uint32_t fb = full0 + static_cast<uint32_t>(stage * sizeof(uint64_t));
+                        uint8_t *st = sm.ring + stage * stage_bytes;
+                        const int x = kb * kTileK;
+                        tma_load_2d_pair(st, tmW, fb, x, n * kTileN + w_off);
+                        uint8_t *sb = st + kSwapStageBytesA;
+                        tma_load_2d_pair(sb, map0, fb, x, rows0);
+                        if (half1 > 0) tma_load_2d_pair(sb + half0 * (kTileK * 2), map1, fb, x, rows1);
+                        ++fills;
+                        if (++stage == stages) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                    }
+                }
+            }
+            for (int s = 0; s < stages; ++s) {
+                const long long n_s = fills / stages + (s < fills % stages ? 1 : 0);
+                if (n_s > 0)
+                    mbar_wait_drain(&empty[s], static_cast<uint32_t>((n_s - 1) & 1), p.wait_limit_ns / 8);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            if (rank == 0) {
+                // ------------------------------------------------ MMA issuer (even CTA only)
+                const uint32_t idesc0 = idesc_bf16_f32(kPairTileM, n0);
+                const uint32_t idesc1 = idesc_bf16_f32(kPairTileM, n1 > 0 ? n1 : 16);
+                const uint32_t b1_off = static_cast<uint32_t>((n0 / 2) * kTileK * 2);
+                int stage = 0;
+                uint32_t phase = 0;
+                uint32_t tile_iter = 0;
+                bool ok = true;
+                UnitCursor uc;
+                while (ok) {
+                    if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+                        break;
+                    const int u = unit_ring[uc.slot];
+                    mbar_arrive(&unit_empty[uc.slot]);
+                    uc.advance();
+                    if (u < 0) break;
+                    int m, g, v0, v1;
+                    tw.unit(u, m, g, v0, v1);
+                    for (int n = v0; ok && n < v1; ++n, ++tile_iter) {
+                        const uint32_t acc = nbuf == 2 ? (tile_iter & 1u) : 0u;
+                        const uint32_t acc_phase = (nbuf == 2 ? (tile_iter >> 1) : tile_iter) & 1u;
+                        if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
+                                               p.wait_limit_ns)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after_sync();
+                        const uint32_t d_tmem = tmem_base + acc * kTileN;
+                        for (int kb = 0; kb < num_kb; ++kb) {
+                            if (!mbar_wait_bounded(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after_sync();
+                            const uint32_t a0 = smem_u32(sm.ring + stage * stage_bytes);
+                            const uint32_t b0 = a0 + kSwapStageBytesA;
+#pragma unroll
+                            for (int kk = 0; kk < kTileK / 16; ++kk) {
+                                const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
+                                umma_bf16_pair(d_tmem, smem_desc_sw128(a0 + kk * 32),
+                                               smem_desc_sw128(b0 + kk * 32), idesc0, accum);
+                                if (n1 > 0)
+                                    umma_bf16_pair(d_tmem + kPairTileM, smem_desc_sw128(a0 + kk * 32),
+                                                   smem_desc_sw128(b0 + b1_off + kk * 32), idesc1, accum);
+                            }
+                            umma_commit_pair_multicast(&empty[stage], 0x3);
+                            if (++stage == stages) {
+                                stage = 0;
+                                phase ^= 1u;
+                            }
+                        }
+                        if (!ok) break;
+                        umma_commit_pair_multicast(&acc_full[acc], 0x3);
+                    }
+                }
+                umma_commit_pair_multicast(sm.drain, 0x3);
+            }
+            mbar_wait_drain(sm.drain, 0, p.wait_limit_ns);
+        }
+    } else {
+        // ---------------------------------------------------------- epilogue (both CTAs)
+        const int ew = warp - 2;                 // 0..7
+        const int sub = warp & 3;                // TMEM sub-partition (lanes 32*sub..+31)
+        const int half = ew >> 2;                // takes chunks half, half + 2, ...
+        const int etid = ew * 32 + lane;         // 0..255
+        const int nch = ng / 32;
+        const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
+        const uint32_t acc_empty0 = mapa_shared(smem_u32(&acc_empty[0]), 0);
+        const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
+        float *xp = sm.xpose + ew * 32 * kSwapXposeStride;
+        float4 *comb = reinterpret_cast<float4 *>(sm.xpose);  // [4][kSwapMaxRows] at a unit's end
+        constexpr int kMaxChunks = kSwapMaxRows / 32 / 2;      // chunks of one warp
+        uint32_t epi_phase = 0;
+        uint32_t tile_iter = 0;
+        bool ok = true;
+        UnitCursor uc;
+        while (ok) {
+            if (!mbar_wait_bounded_cluster(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+                break;
+            const int u = unit_ring[uc.slot];
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive_cluster(unit_empty0 + static_cast<uint32_t>(uc.slot * sizeof(uint64_t)));
+            uc.advance();
+            if (u < 0) break;
+            int m, g, v0, v1;
+            tw.unit(u, m, g, v0, v1);
+            // running statistics of rows (half + 2j)*32 + lane of the group, j < kMaxChunks, over
+            // this warp's 32 vocabulary entries of each tile
+            float scale[kMaxChunks], st_m[kMaxChunks], st_s[kMaxChunks], st_t[kMaxChunks];
+            int st_a[kMaxChunks];
+#pragma unroll
+            for (int j = 0; j < kMaxChunks; ++j) {
+                const int r = m * ng + (half + 2 * j) * 32 + lane;
+                scale[j] = (half + 2 * j < nch && r < rows) ? __ldg(p.inv_rms + r) * kLog2e : 0.f;
+                st_m[j] = -INFINITY;
+                st_s[j] = 0.f;
+                st_t[j] = 0.f;
+                st_a[j] = 0;
+            }
+            for (int n = v0; n < v1; ++n, ++tile_iter) {
+                const uint32_t acc = nbuf == 2 ? (tile_iter & 1u) : 0u;
+                const uint32_t acc_phase = (nbuf == 2 ? (tile_iter >> 1) : tile_iter) & 1u;
+                if (!warp_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after_sync();
+                // the 32 vocabulary entries of this warp's sub-partition
+                const int vbase = n * kTileN + static_cast<int>(rank) * kPairHalfRows + sub * 32;
+                const bool full_tile = vbase + 32 <= p.V;
+#pragma unroll
+                for (int j = 0; j < kMaxChunks; ++j) {
+                    const int c = half + 2 * j;
+                    if (c >= nch) break;
+                    float v[32];
+                    tmem_ld_32x32b_x32(lane_base + acc * kTileN + c * 32, v);
+                    // thread `lane` holds vocabulary entry vbase + lane for rows c*32 + i; write
+                    // it as row `lane` of a block padded to 33 floats a row (bank lane + i: no
+                    // conflict) and read back column `lane` (bank i + lane: no conflict)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) xp[lane * kSwapXposeStride + i] = v[i];
+                    __syncwarp();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = xp[i * kSwapXposeStride + lane];
+                    __syncwarp();
+                    // now v[i] = logit of vocabulary entry vbase + i for row c*32 + lane
+                    if (full_tile)
+                        fold_chunk<true>(v, scale[j], vbase, p.V, st_m[j], st_s[j], st_t[j], st_a[j]);
+                    else
+                        fold_chunk<false>(v, scale[j], vbase, p.V, st_m[j], st_s[j], st_t[j], st_a[j]);
+                }
+                tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(acc_empty0 + acc * static_cast<uint32_t>(sizeof(uint64_t)));
+            }
+            if (!ok) break;
+            // Combine the four sub-partitions' statistics of each row of the group (the
+            // transpose blocks double as the exchange area once every warp is done with them)
+            // and write this CTA's partial.  The epilogue warps meet at an mbarrier rather than a
+            // named barrier, so that a wait that runs out (or another role's abort) can never
+            // leave a warp blocked.
+            if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;
+#pragma unroll
+            for (int j = 0; j < kMaxChunks; ++j) {
+                const int c = half + 2 * j;
+                if (c >= nch) break;
+                comb[sub * kSwapMaxRows + c * 32 + lane] =
+                    make_float4(st_m[j], st_s[j], st_t[j], __int_as_float(st_a[j]));
+            }
+            if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;
+            for (int rl = etid; rl < ng; rl += kEpiThreads) {
+                const int r = m * ng + rl;
+                if (r >= rows) break;
+                float4 acc4 = comb[rl];
+#pragma unroll
+                for (int s4 = 1; s4 < 4; ++s4) acc4 = merge_stat(acc4, comb[s4 * kSwapMaxRows + rl]);
+                p.partials[static_cast<size_t>(r) * p.max_splits + 2 * g + static_cast<int>(rank)] = acc4;
+            }
+            if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;
+        }
+    }
+
+    __syncwarp();
+    tc_fence_before_sync();
+    __syncthreads();
+    cluster_sync();
+    tc_fence_after_sync();
+    if (*abort_flag && threadIdx.x == 0) atomicExch(&p.meta[kMetaStatus], RPD_ERR_TIMEOUT);
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc_pair(tmem_base, kTmemCols);
+    }
+}
+
+// The head kernel: one launch per projection pass, clusters of two CTAs, one CTA per SM.
+__global__ void __launch_bounds__(kHeadKernelThreads, 1)
+    k_head(const __grid_constant__ HeadMaps maps, HeadParams p) {
+    pdl_trigger();  // successors may launch now; they wait for this grid before reading
+    pdl_wait();     // row count, tiling, u and inv_rms come from the preceding kernels
+    const int rows = p.meta[kMetaRows];
+    if (rows == 0) return;  // uniform over the grid: no cluster-wide barrier is left waiting
+    const int mode = p.meta[kMetaHeadMode];
+    const int splits = p.meta[kMetaSplits];
+    extern __shared__ uint8_t smem_raw[];
+    const HeadSmem sm = carve_smem(smem_raw);
+    if (mode == kHeadModePair)
+        head_pair(&maps.u, &maps.w128, p, sm, rows, splits);
+    else if (mode == kHeadModeRowsN)
+        head_swap(maps.u_rows, &maps.w128, p, sm, rows, splits / 2, p.meta[kMetaSwapRows]);
+}
+
 // Per-device one-time settings (the dynamic shared-memory opt-in is a property of the
 // kernel on each device).
 constexpr int kMaxDevices = 64;
-std::atomic<int> g_single_ready[kMaxDevices];
-std::atomic<int> g_pair_ready[kMaxDevices];
-std::atomic<int> g_pair_clusters[kMaxDevices];  // resident pairs + 1 (0: not queried yet)
+std::atomic<int> g_head_ready[kMaxDevices];
+std::atomic<int> g_head_clusters[kMaxDevices];  // resident pairs + 1 (0: not queried yet)
 
 int current_device() {
     int dev = 0;
@@ -614,41 +793,28 @@ int current_device() {
     return dev;
 }
 
-cudaError_t opt_in_smem(const void *kernel, int bytes, std::atomic<int> *ready) {
+cudaError_t opt_in_smem() {
     const int dev = current_device();
     if (dev < 0) return cudaErrorInvalidDevice;
-    if (ready[dev].load(std::memory_order_acquire)) return cudaSuccess;
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) ready[dev].store(1, std::memory_order_release);
+    if (g_head_ready[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(k_head, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kHeadKernelSmemBytes);
+    if (e == cudaSuccess) g_head_ready[dev].store(1, std::memory_order_release);
     return e;
 }
 
 }  // namespace
 
-cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, const HeadParams &p,
-                              int grid, cudaStream_t s) {
-    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(k_head_stats), kHeadSmemBytes,
-                                g_single_ready);
-    if (e != cudaSuccess) return e;
-    return launch_pdl(k_head_stats, dim3(grid), dim3(kHeadThreads), kHeadSmemBytes, s, tmU, tmW, p);
-}
-
-}  // namespace rpd
-
-namespace rpd {
-
-int head_stats_pair_max_clusters() {
+int head_max_clusters() {
     const int dev = current_device();
     if (dev < 0) return 0;
-    const int cached = g_pair_clusters[dev].load(std::memory_order_acquire);
+    const int cached = g_head_clusters[dev].load(std::memory_order_acquire);
     if (cached > 0) return cached - 1;
-    if (opt_in_smem(reinterpret_cast<const void *>(k_head_stats_pair), kPairSmemBytes,
-                    g_pair_ready) != cudaSuccess)
-        return 0;
+    if (opt_in_smem() != cudaSuccess) return 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2);
-    cfg.blockDim = dim3(kHeadThreads);
-    cfg.dynamicSmemBytes = kPairSmemBytes;
+    cfg.blockDim = dim3(kHeadKernelThreads);
+    cfg.dynamicSmemBytes = kHeadKernelSmemBytes;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
@@ -657,20 +823,18 @@ int head_stats_pair_max_clusters() {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, k_head_stats_pair, &cfg) != cudaSuccess) n = 0;
-    g_pair_clusters[dev].store(n + 1, std::memory_order_release);
+    if (cudaOccupancyMaxActiveClusters(&n, k_head, &cfg) != cudaSuccess) n = 0;
+    g_head_clusters[dev].store(n + 1, std::memory_order_release);
     return n;
 }
 
-cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tmW,
-                                   const HeadParams &p, int grid, cudaStream_t s) {
-    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(k_head_stats_pair), kPairSmemBytes,
-                                g_pair_ready);
+cudaError_t launch_head(const HeadMaps &maps, const HeadParams &p, int grid, cudaStream_t s) {
+    cudaError_t e = opt_in_smem();
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kHeadThreads);
-    cfg.dynamicSmemBytes = kPairSmemBytes;
+    cfg.blockDim = dim3(kHeadKernelThreads);
+    cfg.dynamicSmemBytes = kHeadKernelSmemBytes;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -681,7 +845,7 @@ cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tm
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, k_head_stats_pair, tmU, tmW, p);
+    return cudaLaunchKernelEx(&cfg, k_head, maps, p);
 }
 
 }  // namespace rpd

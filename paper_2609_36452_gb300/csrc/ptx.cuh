@@ -161,18 +161,8 @@ __device__ __forceinline__ void st_shared_cluster(uint32_t cluster_addr, int val
 
 // ------------------------------------------------------------------------------ TMA
 
-// 2-D tiled bulk tensor load global -> shared, completing on `bar` (tx bytes = box bytes).
-// x is the innermost (contiguous) coordinate in elements.
-__device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, uint64_t *bar,
-                                            int32_t x, int32_t y) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(smem_dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
-        : "memory");
-}
-
-// As tma_load_2d, for a CTA pair: the completion is signalled on `bar_cluster_addr`, an
+// 2-D tiled bulk tensor load global -> shared for a CTA pair (x is the innermost coordinate in
+// elements); the completion (tx bytes = box bytes) is signalled on `bar_cluster_addr`, an
 // mbarrier in either CTA of the pair (shared::cluster address).
 __device__ __forceinline__ void tma_load_2d_pair(void *smem_dst, const CUtensorMap *map,
                                                  uint32_t bar_cluster_addr, int32_t x, int32_t y) {
@@ -189,23 +179,8 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map) {
 
 // ------------------------------------------------------------------------------ tcgen05
 
-// Allocate `ncols` TMEM columns (power of two >= 32); the address is written to *slot.
-// Executed by one full warp.
-__device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(slot)),
-                 "r"(ncols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-                 : "memory");
-}
-
-// CTA-pair forms: TMEM columns allocated (and freed) in both CTAs of the pair; one warp of
-// each CTA executes them.
+// Allocate `ncols` TMEM columns (a power of two >= 32) in both CTAs of the pair (the address is
+// written to *slot), and free them; one warp of each CTA executes these.
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t *slot, uint32_t ncols) {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(slot)),
@@ -249,27 +224,6 @@ __device__ __forceinline__ void tc_fence_before_sync() {
 
 __device__ __forceinline__ void tc_fence_after_sync() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulation (kind::f16).
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                          uint32_t idesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n"
-        " .reg .pred p;\n"
-        " setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
-        "}\n" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
-// Arrive once on `bar` when every tcgen05.mma issued so far by this thread has completed.
-__device__ __forceinline__ void umma_commit(uint64_t *bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-            smem_u32(bar))
-        : "memory");
 }
 
 // Shared-memory matrix descriptor for a K-major bf16 tile written by TMA with 128-byte

@@ -118,8 +118,8 @@ struct rpd_ctx {
     int tiling = RPD_TILING_AUTO;
     uint64_t wait_limit_ns = kWaitLimitNs;
     bool stall_next = false;  // diagnostics: the next step's head kernels issue no loads
-    CUtensorMap tmU{}, tmW{}, tmW_pair{};
-    int pair_grid = 0;   // CTAs of the CTA-pair head kernel (2 x resident pairs; 0 = none)
+    HeadMaps maps{};     // u (scratch) and W tensor maps of the head kernel
+    int head_grid = 0;   // CTAs of the head kernel: 2 x resident clusters of two, <= SMs
 
     // host-buffer entry point staging: device buffer, and a pinned host copy of its small
     // part (mask, commit, tokens, stats) so that those move in one copy each way
@@ -164,7 +164,8 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
     c->free_scratch();
     const int num_n = (c->V + kTileN - 1) / kTileN;
-    c->max_splits = std::min(num_n, 2 * c->num_sms);
+    // partials per row: a vocabulary split each (pair tiles), two per split (rows on N)
+    c->max_splits = std::min(2 * num_n, 2 * c->num_sms);
     struct {
         void **p;
         size_t bytes;
@@ -199,7 +200,11 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
     c->cap_bn = new_bn;
     c->cap_b = new_b;
     c->cap_rows = static_cast<int>(rows);
-    return encode_bf16_2d(&c->tmU, c->u, static_cast<uint64_t>(rows), c->d, kTileM);
+    int rc = encode_bf16_2d(&c->maps.u, c->u, static_cast<uint64_t>(rows), c->d, kTileM);
+    for (int j = 0; rc == RPD_OK && j < kUMaps; ++j)
+        rc = encode_bf16_2d(&c->maps.u_rows[j], c->u, static_cast<uint64_t>(rows), c->d,
+                            static_cast<uint32_t>(kUBoxRows * (j + 1)));
+    return rc;
 }
 
 cudaEvent_t take_event(rpd_ctx *c) {
@@ -270,7 +275,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
 
     const int bn = B * N;
     const int num_n = (c->V + kTileN - 1) / kTileN;
-    const int pair_slots = c->pair_grid / 2;
+    const int pair_slots = c->head_grid / 2;
     const float hbm_tiles = head_stream_in_tiles(c->V, c->d, c->num_sms);
     // Lazy projection (forced, or chosen on the device per step): a second pass over the band.
     // It is not launched when even the largest possible row count keeps a single pass cheaper.
@@ -281,7 +286,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
     {
         KernelTimer t(c, 0);
         CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
-                         num_n, c->max_splits, c->num_sms, pair_slots, hbm_tiles, c->rule.block,
+                         num_n, c->max_splits, pair_slots, hbm_tiles, c->rule.block,
                          c->projection == RPD_PROJECT_LAZY ? 1 : (lazy ? 2 : 0), c->tiling};
         e = launch_compact(cp, c->stream);
     }
@@ -336,11 +341,8 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             KernelTimer t(c, 1);
             HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits,
                           c->wait_limit_ns, c->stall_next ? 1 : 0};
-            // Both tilings are launched; each reads the choice made on the device for this
-            // pass's row count and the other returns at once.
-            err = launch_head_stats(c->tmU, c->tmW, hp, c->num_sms, c->stream);
-            if (err == cudaSuccess && pair_slots > 0)
-                err = launch_head_stats_pair(c->tmU, c->tmW_pair, hp, c->pair_grid, c->stream);
+            // One launch: the kernel reads the tiling chosen on the device for this pass.
+            err = launch_head(c->maps, hp, c->head_grid, c->stream);
         }
         if (err != cudaSuccess) return err;
         KernelTimer t(c, 2);
@@ -365,7 +367,6 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             bp.theta_c = c->rule.theta_c;
             bp.num_n_tiles = num_n;
             bp.max_splits = c->max_splits;
-            bp.single_slots = c->num_sms;
             bp.pair_slots = pair_slots;
             bp.hbm_tiles = hbm_tiles;
             bp.tiling = c->tiling;
@@ -436,8 +437,13 @@ rpd_ctx *rpd_create(int d, int V, int K, float eps) {
         delete c;
         return nullptr;
     }
-    const int clusters = head_stats_pair_max_clusters();
-    c->pair_grid = 2 * std::min(clusters, c->num_sms / 2);
+    const int clusters = std::min(head_max_clusters(), c->num_sms / 2);
+    if (clusters < 1) {
+        fail(RPD_ERR_UNSUPPORTED, "the head kernel (clusters of two CTAs) cannot be resident on this device");
+        delete c;
+        return nullptr;
+    }
+    c->head_grid = 2 * clusters;
     return c;
 }
 
@@ -451,13 +457,10 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
     if (!pointer_usable(W_head, c->device, false) || !pointer_usable(g_norm, c->device, false))
         return fail(RPD_ERR_INVALID_ARGUMENT,
                     "W_head and g_norm must be device memory on the context's device");
-    CUtensorMap m, m2;
-    int rc = encode_bf16_2d(&m, W_head, static_cast<uint64_t>(c->V), c->d, kTileN);
+    CUtensorMap m2;
+    int rc = encode_bf16_2d(&m2, W_head, static_cast<uint64_t>(c->V), c->d, kPairHalfRows);
     if (rc) return rc;
-    rc = encode_bf16_2d(&m2, W_head, static_cast<uint64_t>(c->V), c->d, kPairHalfRows);
-    if (rc) return rc;
-    c->tmW = m;
-    c->tmW_pair = m2;
+    c->maps.w128 = m2;
     c->W = W_head;
     c->g = g_norm;
     return RPD_OK;
@@ -503,7 +506,7 @@ int rpd_set_projection(rpd_ctx *c, int mode) {
 
 int rpd_set_head_tiling(rpd_ctx *c, int tiling) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
-    if (tiling < RPD_TILING_AUTO || tiling > RPD_TILING_PAIR)
+    if (tiling < RPD_TILING_AUTO || tiling > RPD_TILING_ROWS_N)
         return fail(RPD_ERR_INVALID_ARGUMENT, "unknown head tiling %d", tiling);
     c->tiling = tiling;
     return RPD_OK;

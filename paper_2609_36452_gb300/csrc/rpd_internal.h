@@ -11,23 +11,46 @@
 
 namespace rpd {
 
-// Head-statistics tile: 128 rows (TMEM lanes) x 256 vocabulary columns, K-step 64.
-constexpr int kTileM = 128;
-constexpr int kTileN = 256;
+// Head-statistics tiles (tcgen05 cta_group::2: a cluster of two CTAs, one per SM, M = 256).
+// Pair tiles: 256 rows x 256 vocabulary columns per pair; each CTA stages its own 128 rows of
+// u and 128 rows of W per K-step of 64 (32 KB), 6 stages deep.
+constexpr int kTileM = 128;   // rows of u per CTA (TMEM lanes) and the row padding unit of scratch
+constexpr int kTileN = 256;   // vocabulary entries per tile
 constexpr int kTileK = 64;
-constexpr int kStages = 4;
-constexpr int kHeadThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-5 epilogue
-constexpr int kStageBytesA = kTileM * kTileK * 2;
-constexpr int kStageBytesB = kTileN * kTileK * 2;
-constexpr int kHeadSmemBytes = kStages * (kStageBytesA + kStageBytesB) + 1024 + 256;
-// CTA-pair variant: a pair computes 256 rows x 256 vocabulary columns per tile; each CTA
-// stages its own 128 rows of u and 128 rows of W per K-step (32 KB), 6 stages deep.
 constexpr int kPairTileM = 256;
 constexpr int kPairStages = 6;
 constexpr int kPairHalfRows = 128;
 constexpr int kPairStageBytesA = kPairHalfRows * kTileK * 2;
 constexpr int kPairStageBytesB = kPairHalfRows * kTileK * 2;
-constexpr int kPairSmemBytes = kPairStages * (kPairStageBytesA + kPairStageBytesB) + 1024 + 256;
+// "Rows on N" tiles: a pair multiplies 256 vocabulary entries (128 per CTA, the MMA's M side)
+// by a group of up to 512 projected rows (the N side, in steps of 32), so rows are padded to a
+// multiple of 32 instead of a multiple of 256.  Each CTA stages its 128 head rows (16 KB) and
+// half of the group's rows per K-step; the accumulator of a group of at most 256 rows is
+// double-buffered in TMEM, a larger group uses all 512 columns once.
+constexpr int kSwapMaxRows = 512;
+constexpr int kSwapRowStep = 32;  // N of the M = 256 MMA: a multiple of 32, at least 32
+constexpr int kSwapMaxStages = 8;
+constexpr int kSwapStageBytesA = kPairHalfRows * kTileK * 2;
+constexpr int kSwapStageBudget = 192 * 1024;
+constexpr int kSwapEpiWarps = 8;
+constexpr int kSwapXposeStride = 33;                             // floats per padded row
+constexpr int kSwapXposeBytes = kSwapEpiWarps * 32 * kSwapXposeStride * 4;  // 32 x 32 fp32 per warp
+static_assert(kSwapXposeBytes >= 4 * kSwapMaxRows * 16,
+              "the transpose blocks double as the [sub-partition][row] statistics exchange");
+constexpr int kUBoxRows = 16;  // granularity of a half group's rows (the TMA box heights)
+// Roles: warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-9 epilogue (pair tiles use warps 2-5).
+constexpr int kHeadKernelThreads = 64 + 32 * kSwapEpiWarps;
+constexpr int kHeadBarrierBytes = 512;
+// The operand ring of either tiling, then the rows-on-N transpose blocks.
+constexpr int kHeadRegionBytes = kSwapStageBudget + kSwapXposeBytes;
+static_assert(kPairStages * (kPairStageBytesA + kPairStageBytesB) <= kHeadRegionBytes,
+              "the pair tiles' operand ring fits the region");
+// 1024-byte alignment slack + that region + barriers
+constexpr int kHeadKernelSmemBytes = 1024 + kHeadRegionBytes + kHeadBarrierBytes;
+static_assert(kHeadKernelSmemBytes <= 232448, "dynamic shared memory per CTA");
+// Values of meta[kMetaHeadMode].
+constexpr int kHeadModePair = 2;
+constexpr int kHeadModeRowsN = 3;
 constexpr int kMaxBatch = 128;
 constexpr int kMaxCanvas = 8192;
 constexpr int kScoreThreads = 1024;
@@ -40,13 +63,14 @@ enum MetaIndex : int {
     kMetaRows = 1,     // projected rows R = K * NMT
     kMetaStatus = 2,   // RPD_OK or RPD_ERR_TIMEOUT, latched by kernels
     kMetaSplits = 3,   // vocabulary splits G chosen for the head kernel
-    kMetaHeadMode = 4, // 1: single-CTA head tiles, 2: CTA-pair head tiles
+    kMetaHeadMode = 4, // kHeadModePair or kHeadModeRowsN: the pass's head tiling
     kMetaSel = 5,      // positions projected by the current pass
     kMetaLayer0 = 6,   // first window layer of the current pass (rows are layer-major)
     kMetaRowsTotal = 7,// rows projected by all passes of this step
     kMetaLazy = 8,     // 1 when this step projects lazily (two passes)
     kMetaUnitNext = 9, // next head work unit to claim (zeroed before each projection pass)
     kMetaMergeDone = 10, // CTAs that finished the fused merge-and-score (zeroed per step)
+    kMetaSwapRows = 11,  // rows per row group of the "rows on N" tiling (mode 3)
     kMetaWords = 16
 };
 
@@ -59,9 +83,8 @@ struct CompactParams {
     int B, N, K;
     int num_n_tiles;      // ceil(V / kTileN)
     int max_splits;       // capacity of the partial-statistics buffer per row
-    int single_slots;     // CTAs of the single-CTA head kernel
-    int pair_slots;       // CTA pairs of the pair head kernel (0: pair tiles unavailable)
-    float hbm_tiles;      // time to stream the head once, in single-CTA tile times
+    int pair_slots;       // CTA pairs of the head kernel
+    float hbm_tiles;      // time to stream the head once, in pair-tile units (see below)
     int block;            // 0: every masked position; > 0: only each canvas's active block
     int lazy;             // 0: all window layers; 1: lazy; 2: lazy when it is estimated cheaper
     int tiling;           // RPD_TILING_*: head tiling, or 0 to choose per pass
@@ -93,17 +116,23 @@ struct BandParams {
     int32_t *band_off;         // out: [B+1] first band entry of each canvas
     int B, N, K;
     float theta_c;
-    int num_n_tiles, max_splits, single_slots, pair_slots;
+    int num_n_tiles, max_splits, pair_slots;
     float hbm_tiles;
     int tiling;
     float tau[kMaxBatch];
 };
 
-// Relative cost of a CTA-pair tile (256 rows on two SMs) against a single-CTA tile (128 rows
-// on one SM): measured per-SM throughput of the pair form on GB300 at the LLaDA head shape.
+// Costs of the tiling choice are in units of one 128-row x 256-entry tile's MMA work on one
+// SM.  A pair tile (256 rows on two SMs) costs kPairTileCost per SM: the measured per-SM rate
+// of the pair form on GB300 at the LLaDA head shape against that unit's nominal rate.
 constexpr float kPairTileCost = 0.88f;
-// Per-SM rate of the single-CTA tile and the sustained HBM read rate used by the tiling
-// choice (GB300 measurements; only their ratio matters).
+// "Rows on N" tiles: extra time of a group over 256 rows, whose epilogue cannot overlap the
+// next tile's MMAs (single-buffered TMEM), and the time per unit of operand bytes an SM
+// receives, relative to the 384 rows' worth of a 128 x 256 tile.
+constexpr float kSwapSingleBufferCost = 1.08f;
+constexpr float kSwapFeedCost = 1.0f;
+// Per-SM MMA rate of the unit tile and the sustained HBM read rate used by the tiling choice
+// (GB300 measurements; only their ratio matters).
 constexpr double kSingleTileFlopsPerSm = 1.1e13;
 constexpr double kHeadStreamBytesPerSec = 6.5e12;
 
@@ -131,7 +160,7 @@ struct HeadParams {
     int stall;               // diagnostics: issue no loads (the waits run out)
 };
 
-// Time to stream the head once, in units of one single-CTA tile's MMA time.
+// Time to stream the head once, in units of one 128 x 256 tile's MMA time on one SM.
 inline float head_stream_in_tiles(int V, int d, int num_sms) {
     (void)num_sms;
     const double t_hbm = 2.0 * V * static_cast<double>(d) / kHeadStreamBytesPerSec;
@@ -224,13 +253,22 @@ inline bool pointer_usable(const void *p, int device, bool host_mapped_ok) {
 
 cudaError_t launch_compact(const CompactParams &p, cudaStream_t s);
 cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s);
-cudaError_t launch_head_stats(const CUtensorMap &tmU, const CUtensorMap &tmW, const HeadParams &p,
-                              int grid, cudaStream_t s);
-// tmU/tmW boxes: 64 x 128 rows.  grid = 2 x (pairs); clusters of 2 CTAs.
-cudaError_t launch_head_stats_pair(const CUtensorMap &tmU, const CUtensorMap &tmW,
-                                   const HeadParams &p, int grid, cudaStream_t s);
-// Largest number of CTA pairs of the pair kernel that can be resident at once.
-int head_stats_pair_max_clusters();
+// Tensor maps of the head kernel's operands (128-byte swizzling, K boxes of 64): u in boxes of
+// 128 rows (pair tiles) and, for the rows-on-N tiles, in boxes of 16, 32, ..., 128 rows (one
+// per half-group height, so that a stage copies each MMA's share of u with one instruction:
+// the TMA unit's time per copy, not its bytes, bounded a stage built from 16-row boxes); W in
+// boxes of 128 rows.
+constexpr int kUMaps = kPairHalfRows / kUBoxRows;  // box heights kUBoxRows * (1 .. kUMaps)
+struct HeadMaps {
+    CUtensorMap u;                // box 64 x 128 rows
+    CUtensorMap w128;             // box 64 x 128 rows of W
+    CUtensorMap u_rows[kUMaps];   // u_rows[j]: box 64 x kUBoxRows*(j+1) rows
+};
+// The head kernel (every tiling; the pass's choice is read from the meta words), launched as
+// `grid` CTAs in clusters of two, one per SM.
+cudaError_t launch_head(const HeadMaps &maps, const HeadParams &p, int grid, cudaStream_t s);
+// Largest number of clusters of the head kernel that can be resident at once.
+int head_max_clusters();
 cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,
                          int grid, cudaStream_t s);
 cudaError_t launch_band(const BandParams &p, cudaStream_t s);

@@ -71,7 +71,7 @@ struct DeviceSetup {
     int device = 0;
     uint8_t *arena = nullptr;  // device address of g_noalloc_arena on this device
     int num_sms = 0;
-    int pair_grid = 0;         // CTAs of the CTA-pair head kernel (same choice as rpd_step)
+    int head_grid = 0;         // CTAs of the head kernel (same choice as rpd_step)
 };
 
 std::mutex g_setup_mutex;
@@ -131,7 +131,10 @@ int setup_device(DeviceSetup **out) {
         s.device = dev;
         s.arena = static_cast<uint8_t *>(ptr);
         s.num_sms = sms;
-        s.pair_grid = 2 * std::min(head_stats_pair_max_clusters(), sms / 2);
+        const int clusters = std::min(head_max_clusters(), sms / 2);
+        if (clusters < 1)
+            return na_fail(RPD_ERR_UNSUPPORTED, "the head kernel cannot be resident on this device");
+        s.head_grid = 2 * clusters;
         s.ready = true;
     }
     *out = &s;
@@ -194,24 +197,26 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     int32_t *canvas_off = reinterpret_cast<int32_t *>(A + kOffCanvasOff);
     int32_t *meta = reinterpret_cast<int32_t *>(A + kOffMeta);
 
-    // Same head-kernel configuration as rpd_step (both tilings, chosen on the device).
-    const int pair_slots = dev->pair_grid / 2;
-    CUtensorMap tmU, tmW, tmW_pair;
-    if (!encode_tile_map(&tmU, u, kNaMaxRows, static_cast<uint64_t>(d), kTileM) ||
-        !encode_tile_map(&tmW, W_head, static_cast<uint64_t>(V), static_cast<uint64_t>(d), kTileN) ||
-        !encode_tile_map(&tmW_pair, W_head, static_cast<uint64_t>(V), static_cast<uint64_t>(d),
-                         kPairHalfRows))
-        return na_fail(RPD_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+    // Same head-kernel configuration as rpd_step (tiling chosen on the device).
+    const int pair_slots = dev->head_grid / 2;
+    HeadMaps maps;
+    bool maps_ok = encode_tile_map(&maps.u, u, kNaMaxRows, static_cast<uint64_t>(d), kTileM) &&
+                   encode_tile_map(&maps.w128, W_head, static_cast<uint64_t>(V),
+                                   static_cast<uint64_t>(d), kPairHalfRows);
+    for (int j = 0; maps_ok && j < kUMaps; ++j)
+        maps_ok = encode_tile_map(&maps.u_rows[j], u, kNaMaxRows, static_cast<uint64_t>(d),
+                                  static_cast<uint32_t>(kUBoxRows * (j + 1)));
+    if (!maps_ok) return na_fail(RPD_ERR_CUDA, "cuTensorMapEncodeTiled failed");
 
     const int num_n = (V + kTileN - 1) / kTileN;
-    int splits = num_n < 2 * dev->num_sms ? num_n : 2 * dev->num_sms;
+    int splits = 2 * num_n < 2 * dev->num_sms ? 2 * num_n : 2 * dev->num_sms;
     if (splits > kNaMaxSplits) splits = kNaMaxSplits;
 
     // The per-step count/status words must start from zero on every call.
     cudaError_t e = cudaMemsetAsync(meta, 0, kMetaWords * 4, stream);
     if (e == cudaSuccess) {
         CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n, splits,
-                         dev->num_sms, pair_slots, head_stream_in_tiles(V, d, dev->num_sms),
+                         pair_slots, head_stream_in_tiles(V, d, dev->num_sms),
                          rule.block, 0, RPD_TILING_AUTO};
         e = launch_compact(cp, stream);
     }
@@ -223,9 +228,7 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     }
     if (e == cudaSuccess) {
         HeadParams hp{inv_rms, partials, meta, V, d, splits, kWaitLimitNs, 0};
-        e = launch_head_stats(tmU, tmW, hp, dev->num_sms, stream);
-        if (e == cudaSuccess && pair_slots > 0)
-            e = launch_head_stats_pair(tmU, tmW_pair, hp, dev->pair_grid, stream);
+        e = launch_head(maps, hp, dev->head_grid, stream);
     }
     if (e == cudaSuccess) {
         // the merge's last CTA scores the canvas (N <= kNaMaxN <= kFuseScoreMaxN), as rpd_step does

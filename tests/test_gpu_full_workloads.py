@@ -1,13 +1,15 @@
 """Full-size workloads that the fp64 oracle cannot evaluate row for row in seconds.
 
 * Batched serving: 8 canvases x 1024 positions, K = 6, LLaDA-8B head, 30-100% masked
-  (~32k projected rows).  Sampled positions of every canvas are projected by the oracle and
-  compared score by score; the commitment of every canvas is checked by replaying the
-  oracle's rule on the GPU's own scores (a property that holds at any size).
+  (~32k projected rows).  Two whole canvases (about 5k rows each) are compared with the whole
+  oracle step, output by output; sampled positions of every canvas, and the positions of the
+  rows on both sides of every L2-band boundary of the head kernel's work walk, are projected
+  by the oracle and compared score by score; the commitment of every canvas is also checked
+  by replaying the oracle's rule on the GPU's own scores.
 * Decode trajectory at the LLaDA-8B head shape: at every step the invariants, the commit
-  rule replayed on the GPU's scores, two sampled positions against the oracle, and the same
-  commits with the projection chosen per step on the device; the full oracle at the first,
-  a middle and the last step.
+  rule replayed on the GPU's scores, the same commits with the projection chosen per step on
+  the device, and the whole oracle step (every projected row, the commit set) compared
+  output by output.
 """
 
 import numpy as np
@@ -17,6 +19,7 @@ import torch
 import workloads as WL
 from oracle import rpd_oracle as O
 from tests.gpu_util import DeviceRunner, bits
+from tests.oracle_pool import oracle_steps
 from tests.parity import DELTA, compare_rows, compare_step, replay_commit_rule
 
 pytestmark = pytest.mark.gpu
@@ -52,6 +55,16 @@ def test_batched_serving_full():
     for b in range(B):
         idx = np.nonzero(case["mask"][b].numpy())[0]
         samples[b] = [int(i) for i in gen.choice(idx, size=min(3, len(idx)), replace=False)]
+    # Rows on both sides of every boundary between L2 bands of the head kernel's work walk
+    # (rows are layer-major over the canvases' masked positions in order; a band covers
+    # 16 tiles of 256 rows), and the positions they belong to.
+    order = [(b, int(i)) for b in range(B) for i in np.nonzero(case["mask"][b].numpy())[0]]
+    nmt = len(order)
+    R = K * nmt
+    for r in [x for j in range(1, R // 4096 + 1) for x in (4096 * j - 1, 4096 * j) if x < R]:
+        b, i = order[r % nmt]
+        if i not in samples[b]:
+            samples[b].append(i)
     picks = [(b, i) for b in range(B) for i in samples[b]]
     rows = torch.stack([case["hidden"][:, b, i] for b, i in picks])    # [P][K][d]
     readouts = dict(zip(picks, oracle_rows(rows, case["g"], case["W"], case["eps"])))
@@ -77,6 +90,15 @@ def test_batched_serving_full():
         # sampled positions against the oracle
         ref_rows = {i: readouts[(b, i)] for i in samples[b]}
         compare_rows(ref_rows, got, samples[b], K)
+    # Whole canvases against the whole oracle step: every projected row of the canvas and its
+    # commit set (the canvases are independent, so the oracle runs each on its own).
+    counts = [int(case["mask"][b].sum()) for b in range(B)]
+    whole = sorted(range(B), key=lambda b: abs(counts[b] - 850))[:2]
+    tasks = [(bits(case["hidden"][:, b]), case["mask"][b].numpy(), case["eps"], case["tau"][b],
+              case["budget"][b], "llada") for b in whole]
+    for b, ref in zip(whole, oracle_steps(case["V"], case["d"], 5, tasks)):
+        rep = compare_step(ref, outs[b])
+        print(f"canvas {b}: {K * counts[b]} rows against the whole oracle step: {rep}")
 
 
 @pytest.fixture(scope="module")
@@ -139,9 +161,11 @@ def test_llada_trajectory(traj_head):
     for t, (cv, m, got) in enumerate(steps):
         mine = [i for tt, i in samples if tt == t]
         compare_rows({i: readouts[(t, i)] for i in mine}, got, mine, K)
-    for t in sorted({0, len(steps) // 2, len(steps) - 1}):
-        cv, m, got = steps[t]
-        ref = O.rpd_step(bits(cv.hidden), m.numpy(), bits(g), bits(W), 1e-6, 0.9, 1.0, "llada")
-        compare_step(ref, got)
-        checked.append(t)
-    print("trajectory steps", len(steps), "oracle-checked", checked)
+    # the whole oracle step at every step of the trajectory (worker processes; each draws the
+    # same head from its seed)
+    tasks = [(bits(cv.hidden), m.numpy(), 1e-6, 0.9, 1.0, "llada") for cv, m, got in steps]
+    refs = oracle_steps(V, WL.LLADA_D, 4, tasks)
+    for t, ((cv, m, got), ref) in enumerate(zip(steps, refs)):
+        rep = compare_step(ref, got)
+        checked.append((t, rep.n_masked, len(rep.near_threshold)))
+    print("trajectory steps", len(steps), "oracle-checked (step, masked, near-threshold)", checked)

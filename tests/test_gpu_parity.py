@@ -107,13 +107,13 @@ def test_ragged_shapes(d, V, K, N, frac):
     print(rep)
 
 
-@pytest.mark.parametrize("tiling", ["single", "pair"])
+@pytest.mark.parametrize("tiling", ["pair", "rows_n"])
 @pytest.mark.parametrize("d,V,K,N,frac", [
-    (256, 4100, 3, 100, 1.0),    # 300 rows: ragged last row tile of either tiling
+    (256, 4100, 3, 100, 1.0),    # 300 rows: ragged last tile / one 320-row group
     (4096, 1280, 3, 50, 1.0),    # 150 rows, 64 K-blocks
     (200, 1000, 2, 77, 0.7),     # ragged K-block and vocabulary tile, ~108 rows
-    (128, 4100, 5, 300, 1.0),    # 1500 rows: 12 single / 6 pair row tiles
-    (64, 512, 4, 128, 1.0),      # 512 rows: whole row tiles only
+    (128, 4100, 5, 300, 1.0),    # 1500 rows: 6 pair row tiles / 3 groups of 512
+    (64, 512, 4, 128, 1.0),      # 512 rows: whole tiles / one full group
 ])
 def test_head_tilings_match_oracle(tiling, d, V, K, N, frac):
     """Both head tilings, forced, on the same inputs; each is compared with the oracle
@@ -129,8 +129,40 @@ def test_head_tilings_match_oracle(tiling, d, V, K, N, frac):
     print(compare_step(ref, got))
 
 
+@pytest.mark.parametrize("tiling", ["pair", "rows_n"])
+@pytest.mark.parametrize("rows", [1, 64, 127, 128, 129, 257, 320, 383, 384, 385, 513, 769, 832,
+                                  895, 896, 897, 1023, 1025])
+def test_row_counts_around_tile_boundaries(tiling, rows):
+    """Row counts 256q + {1, 64, 127, 128, 129} (and around the 512-row group of the rows-on-N
+    tiling) on both tilings: one window layer, so the pass projects exactly `rows` rows; every
+    output is compared with the oracle."""
+    case = small_case(700 + rows, K=1, N=rows, d=192, V=2100, w_std=0.08)
+    runner = DeviceRunner(case["W"], case["g"], 1, case["eps"], rule=case["rule"])
+    try:
+        runner.ctx.set_head_tiling(tiling)
+        got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+    finally:
+        runner.close()
+    assert got["stats"]["n_rows"] == rows
+    print(compare_step(oracle_step(case), got))
+
+
+@pytest.mark.parametrize("K,N", [(4, 70), (4, 107), (4, 128), (2, 300)])
+def test_rows_n_groups_with_window_layers(K, N):
+    """The rows-on-N tiling with several window layers (rows are layer-major, so a group mixes
+    layers and positions): 280, 428 (two groups of 224 or one of 448), 512 and 600 rows."""
+    case = small_case(900 + K * N, K=K, N=N, d=256, V=4100, w_std=0.08)
+    runner = DeviceRunner(case["W"], case["g"], K, case["eps"], rule=case["rule"])
+    try:
+        runner.ctx.set_head_tiling("rows_n")
+        got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+    finally:
+        runner.close()
+    print(compare_step(oracle_step(case), got))
+
+
 def test_many_row_tiles_in_bands():
-    """5100 rows at d = 4096: 20 CTA-pair row tiles (40 single-CTA ones) of 1-2 MB of u each,
+    """5100 rows at d = 4096: 20 CTA-pair row tiles (10 rows-on-N groups) of 2-4 MB of u each,
     more than the head kernels keep in one L2 band of work units, so every row of the second
     band comes from the band-ordered unit walk.  Every output is compared with the oracle."""
     case = small_case(301, K=5, N=1020, d=4096, V=4100, w_std=0.02)
@@ -600,15 +632,17 @@ def test_batched_heterogeneous_lengths():
 
 # ----------------------------------------------------------------------------- failure detection
 
-@pytest.mark.parametrize("N,K", [(256, 4), (32, 2)])   # CTA-pair and single-CTA head tilings
-def test_stalled_head_reports_timeout_and_context_recovers(N, K):
-    """A step whose head kernels issue no loads: their bounded waits run out, the step reports
+@pytest.mark.parametrize("N,K,tiling", [(256, 4, "pair"), (32, 2, "rows_n"), (150, 4, "rows_n")])
+def test_stalled_head_reports_timeout_and_context_recovers(N, K, tiling):
+    """A step whose head kernel issues no loads: its bounded waits run out, the step reports
     RPD_ERR_TIMEOUT in rpd_stats.status without faulting or hanging, and the next step on the
-    same context is correct again."""
+    same context is correct again (both tilings; 600 rows make one single-buffered rows-on-N
+    group)."""
     import paper_2609_36452_gb300 as rpd
     case = small_case(301 + N, K=K, N=N)
     runner = DeviceRunner(case["W"], case["g"], K)
     try:
+        runner.ctx.set_head_tiling(tiling)
         runner.ctx.set_wait_limit(20000)          # 20 ms
         runner.ctx.inject_stall()
         bad = runner.step(case["hidden"], case["mask"], 0.9, 1.0)
