@@ -20,7 +20,10 @@ namespace {
 constexpr int kCompactThreads = 1024;
 constexpr int kCompactItems = 4;
 
-__global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p) {
+// At most 48 registers a thread: the CTA then needs 48 K of an SM's 64 K registers, so it can
+// start (launched early, waiting on its predecessor) beside one CTA of the previous step's merge
+// instead of waiting for an SM to empty.
+__global__ void __maxnreg__(48) k_compact(CompactParams p) {
     __shared__ int warp_sum[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int block_lo[kMaxBatch];  // RPD-block: first position of each canvas's active block
@@ -85,25 +88,27 @@ __global__ void __launch_bounds__(kCompactThreads, 1) k_compact(CompactParams p)
     // the earlier layers of an assumed band fraction) are estimated cheaper than one pass
     // over all layers.
     __shared__ int lazy_on;
+    __shared__ HeadPlan plan;
     const long long all_rows = static_cast<long long>(p.K) * carry;
-    if (p.lazy == 2 && p.K > 1) {
-        int m_, s_, n_;
-        const float e_all = choose_head_tiling(all_rows, p.num_n_tiles, p.max_splits,
-                                               p.pair_slots, p.hbm_tiles, p.tiling, m_, s_, n_);
-        const float e_fin = choose_head_tiling(carry, p.num_n_tiles, p.max_splits,
-                                               p.pair_slots, p.hbm_tiles, p.tiling, m_, s_, n_);
-        const long long guess = static_cast<long long>(kLazyBandGuess * (p.K - 1) * carry);
-        const float e_band = choose_head_tiling(guess, p.num_n_tiles, p.max_splits,
-                                                p.pair_slots, p.hbm_tiles, p.tiling, m_, s_, n_);
-        if (tid == 0) lazy_on = (e_fin + e_band < e_all) ? 1 : 0;
-    } else if (tid == 0) {
-        lazy_on = (p.lazy == 1 && p.K > 1) ? 1 : 0;
+    if (warp == 0) {
+        int lz = (p.lazy == 1 && p.K > 1) ? 1 : 0;
+        if (p.lazy == 2 && p.K > 1) {
+            const long long guess = static_cast<long long>(kLazyBandGuess * (p.K - 1) * carry);
+            const float e_all = lookup_plan(all_rows, p.plan, p.plan_rows, p.plan_in).est;
+            const float e_fin = lookup_plan(carry, p.plan, p.plan_rows, p.plan_in).est;
+            const float e_band = lookup_plan(guess, p.plan, p.plan_rows, p.plan_in).est;
+            lz = (e_fin + e_band < e_all) ? 1 : 0;
+        }
+        const HeadPlan hp = lookup_plan(lz ? static_cast<long long>(carry) : all_rows, p.plan,
+                                        p.plan_rows, p.plan_in);
+        if (lane == 0) {
+            lazy_on = lz;
+            plan = hp;
+        }
     }
     __syncthreads();
     const long long rows = lazy_on ? static_cast<long long>(carry) : all_rows;
-    int mode, splits, swap_rows;
-    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.pair_slots,
-                       p.hbm_tiles, p.tiling, mode, splits, swap_rows);
+    const int mode = plan.mode, splits = plan.splits, swap_rows = plan.swap_rows;
     if (tid == 0) {
         p.canvas_off[p.B] = carry;
         p.meta[kMetaSwapRows] = swap_rows;

@@ -21,7 +21,7 @@
 //                padded to a multiple of 32), so that a pass whose row count is not a multiple
 //                of 256 pads by at most 31 rows per group.
 // Roles: warp 0 TMA producer (one thread), warp 1 TMEM owner (512 columns) and MMA issuer
-// (one thread, even CTA), warps 2-5 (2-9 for rows on N) epilogue.  Every wait is bounded; a
+// (one thread, even CTA), warps 2-5 epilogue.  Every wait is bounded; a
 // timeout latches RPD_ERR_TIMEOUT in the step's status word and the CTA drains and exits.
 #include <atomic>
 
@@ -119,18 +119,6 @@ __device__ __forceinline__ void fold_chunk(float (&x)[32], float scale, int col0
     }
 }
 
-// Wait of a whole warp for a phase that takes long to complete (an accumulator): one lane polls,
-// the others wait at the warp barrier instead of competing for issue slots with the producer
-// and MMA threads, then every lane observes the completed phase itself (acquire).
-__device__ __forceinline__ bool warp_wait_bounded(uint64_t *bar, uint32_t parity,
-                                                  volatile int *abort, uint64_t limit_ns) {
-    int ok = 1;
-    if ((threadIdx.x & 31) == 0) ok = mbar_wait_bounded(bar, parity, abort, limit_ns) ? 1 : 0;
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    if (ok) mbar_try_wait(smem_u32(bar), parity);
-    return ok != 0;
-}
-
 // Combine two partial statistics (same rule as the merge kernel's): m = max, alpha =
 // 2^(m_j - m), s = sum alpha s_j, t = sum alpha (t_j + (m_j - m) s_j), argmax the lowest index
 // attaining m.
@@ -146,12 +134,11 @@ __device__ __forceinline__ float4 merge_stat(float4 x, float4 y) {
                        __int_as_float(a));
 }
 
-// Shared memory of the head kernel: the operand ring, the rows-on-N transpose blocks, then the
-// barriers.
+// Shared memory of the head kernel: the operand ring (and for rows on N the transpose blocks
+// and running statistics), then the barriers.
 struct HeadSmem {
     uint8_t *ring;            // 1024-byte aligned
-    float *xpose;             // rows on N: [kSwapEpiWarps][32][33] transpose blocks, and at the
-                              // end of a unit the [4][kSwapMaxRows] statistics exchange
+
     uint64_t *full;           // [kSwapMaxStages] TMA -> MMA (in the even CTA for pair tilings)
     uint64_t *empty;          // [kSwapMaxStages] MMA -> TMA
     uint64_t *acc_full;       // [2] MMA -> epilogue
@@ -169,8 +156,7 @@ __device__ __forceinline__ HeadSmem carve_smem(uint8_t *raw) {
     HeadSmem s;
     uint8_t *base = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    s.ring = base;
-    s.xpose = reinterpret_cast<float *>(base + kSwapStageBudget);
+    s.ring = base;  // the rows-on-N tiles place their transpose blocks and statistics after their ring
     uint64_t *bars = reinterpret_cast<uint64_t *>(base + kHeadRegionBytes);
     s.full = bars;
     s.empty = bars + kSwapMaxStages;
@@ -396,7 +382,7 @@ __device__ __forceinline__ void head_pair(const CUtensorMap *tmU, const CUtensor
             for (int n = n0; n < n1; ++n, ++tile_iter) {
                 const uint32_t acc = tile_iter & 1u;
                 const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                if (!warp_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
+                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
                     ok = false;
                     break;
                 }
@@ -436,7 +422,7 @@ __device__ __forceinline__ void head_pair(const CUtensorMap *tmU, const CUtensor
     }
 }
 
-// Barrier of the rows-on-N epilogue's 256 threads: every thread arrives (release) and waits
+// Barrier of the rows-on-N epilogue's threads: every thread arrives (release) and waits
 // for the phase (acquire), bounded like every other wait.  Returns false if it gave up.
 __device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, volatile int *abort,
                                          uint64_t limit_ns) {
@@ -454,12 +440,13 @@ __device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, volatil
 // CTA's.  A group of more than 256 rows is issued as two MMAs (N = 256 and N = G_r - 256,
 // TMEM columns [0, 256) and [256, G_r)); a group of at most 256 rows is double-buffered in
 // TMEM.  So CTA r's TMEM holds logits for 128 vocabulary entries (lanes) x the group's rows
-// (columns): per row the softmax statistics reduce across lanes.  The epilogue (8 warps; the
-// two warps that share a TMEM sub-partition take alternate 32-column chunks) loads a 32 x 32
+// (columns): per row the softmax statistics reduce across lanes.  The epilogue (4 warps, one
+// per TMEM sub-partition, each taking every 32-column chunk of its lanes) loads a 32 x 32
 // block, transposes it through shared memory so that each thread holds one row's 32
-// vocabulary entries, and folds them into that row's running statistics.  At the end of a
-// work unit the four sub-partitions' statistics of each row are combined through shared
-// memory and each CTA writes one partial per row (the merge sees 2 partials per split).
+// vocabulary entries, and folds them into that row's running statistics (per sub-partition,
+// in shared memory).  At the end of a work unit the four sub-partitions' statistics of each
+// row are combined and each CTA writes one partial per row (the merge sees 2 partials per
+// split).
 // Each MMA's share of u in a stage is one TMA copy, from the tensor map whose box has that
 // share's height (16 to 128 rows).
 __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps] */,
@@ -479,8 +466,11 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
     const int nbuf = ng <= kPairTileM ? 2 : 1;
     const int stage_b = (ng / 2) * kTileK * 2;
     const int stage_bytes = kSwapStageBytesA + stage_b;
-    int stages = kSwapStageBudget / stage_bytes;
+    // region: operand ring (as many stages as fit), transpose blocks, statistics [4][ng]
+    int stages = (kHeadRegionBytes - kSwapXposeBytes - 4 * ng * 16) / stage_bytes;
     stages = stages < kSwapMaxStages ? stages : kSwapMaxStages;
+    float *xpose = reinterpret_cast<float *>(sm.ring + stages * stage_bytes);
+    float4 *stats = reinterpret_cast<float4 *>(sm.ring + stages * stage_bytes + kSwapXposeBytes);
     constexpr int kEpiThreads = 32 * kSwapEpiWarps;
 
     if (threadIdx.x == 0) {
@@ -650,20 +640,18 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
         }
     } else {
         // ---------------------------------------------------------- epilogue (both CTAs)
-        const int ew = warp - 2;                 // 0..7
         const int sub = warp & 3;                // TMEM sub-partition (lanes 32*sub..+31)
-        const int half = ew >> 2;                // takes chunks half, half + 2, ...
-        const int etid = ew * 32 + lane;         // 0..255
+        const int etid = (warp - 2) * 32 + lane; // 0 .. kEpiThreads-1
         const int nch = ng / 32;
         const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
         const uint32_t acc_empty0 = mapa_shared(smem_u32(&acc_empty[0]), 0);
         const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
-        float *xp = sm.xpose + ew * 32 * kSwapXposeStride;
-        float4 *comb = reinterpret_cast<float4 *>(sm.xpose);  // [4][kSwapMaxRows] at a unit's end
-        constexpr int kMaxChunks = kSwapMaxRows / 32 / 2;      // chunks of one warp
+        float *xp = xpose + (warp - 2) * 32 * kSwapXposeStride;
+        const float4 kEmpty = make_float4(-INFINITY, 0.f, 0.f, __int_as_float(0));
+        for (int i = etid; i < 4 * ng; i += kEpiThreads) stats[i] = kEmpty;
         uint32_t epi_phase = 0;
         uint32_t tile_iter = 0;
-        bool ok = true;
+        bool ok = epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns);
         UnitCursor uc;
         while (ok) {
             if (!mbar_wait_bounded_cluster(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
@@ -676,23 +664,10 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
             if (u < 0) break;
             int m, g, v0, v1;
             tw.unit(u, m, g, v0, v1);
-            // running statistics of rows (half + 2j)*32 + lane of the group, j < kMaxChunks, over
-            // this warp's 32 vocabulary entries of each tile
-            float scale[kMaxChunks], st_m[kMaxChunks], st_s[kMaxChunks], st_t[kMaxChunks];
-            int st_a[kMaxChunks];
-#pragma unroll
-            for (int j = 0; j < kMaxChunks; ++j) {
-                const int r = m * ng + (half + 2 * j) * 32 + lane;
-                scale[j] = (half + 2 * j < nch && r < rows) ? __ldg(p.inv_rms + r) * kLog2e : 0.f;
-                st_m[j] = -INFINITY;
-                st_s[j] = 0.f;
-                st_t[j] = 0.f;
-                st_a[j] = 0;
-            }
             for (int n = v0; n < v1; ++n, ++tile_iter) {
                 const uint32_t acc = nbuf == 2 ? (tile_iter & 1u) : 0u;
                 const uint32_t acc_phase = (nbuf == 2 ? (tile_iter >> 1) : tile_iter) & 1u;
-                if (!warp_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
+                if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
                     ok = false;
                     break;
                 }
@@ -700,10 +675,8 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                 // the 32 vocabulary entries of this warp's sub-partition
                 const int vbase = n * kTileN + static_cast<int>(rank) * kPairHalfRows + sub * 32;
                 const bool full_tile = vbase + 32 <= p.V;
-#pragma unroll
-                for (int j = 0; j < kMaxChunks; ++j) {
-                    const int c = half + 2 * j;
-                    if (c >= nch) break;
+#pragma unroll 1
+                for (int c = 0; c < nch; ++c) {
                     float v[32];
                     tmem_ld_32x32b_x32(lane_base + acc * kTileN + c * 32, v);
                     // thread `lane` holds vocabulary entry vbase + lane for rows c*32 + i; write
@@ -716,37 +689,39 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                     for (int i = 0; i < 32; ++i) v[i] = xp[i * kSwapXposeStride + lane];
                     __syncwarp();
                     // now v[i] = logit of vocabulary entry vbase + i for row c*32 + lane
+                    const int rl = c * 32 + lane;
+                    const int r = m * ng + rl;
+                    const float scale = r < rows ? __ldg(p.inv_rms + r) * kLog2e : 0.f;
+                    float4 st = stats[sub * ng + rl];
+                    int a = __float_as_int(st.w);
                     if (full_tile)
-                        fold_chunk<true>(v, scale[j], vbase, p.V, st_m[j], st_s[j], st_t[j], st_a[j]);
+                        fold_chunk<true>(v, scale, vbase, p.V, st.x, st.y, st.z, a);
                     else
-                        fold_chunk<false>(v, scale[j], vbase, p.V, st_m[j], st_s[j], st_t[j], st_a[j]);
+                        fold_chunk<false>(v, scale, vbase, p.V, st.x, st.y, st.z, a);
+                    st.w = __int_as_float(a);
+                    stats[sub * ng + rl] = st;
                 }
                 tc_fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_cluster(acc_empty0 + acc * static_cast<uint32_t>(sizeof(uint64_t)));
             }
             if (!ok) break;
-            // Combine the four sub-partitions' statistics of each row of the group (the
-            // transpose blocks double as the exchange area once every warp is done with them)
-            // and write this CTA's partial.  The epilogue warps meet at an mbarrier rather than a
-            // named barrier, so that a wait that runs out (or another role's abort) can never
-            // leave a warp blocked.
-            if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;
-#pragma unroll
-            for (int j = 0; j < kMaxChunks; ++j) {
-                const int c = half + 2 * j;
-                if (c >= nch) break;
-                comb[sub * kSwapMaxRows + c * 32 + lane] =
-                    make_float4(st_m[j], st_s[j], st_t[j], __int_as_float(st_a[j]));
-            }
+            // Combine the four sub-partitions' statistics of each row of the group, write this
+            // CTA's partial and reset the entries for the next unit.  The epilogue warps meet at
+            // an mbarrier rather than a named barrier, so that a wait that runs out (or another
+            // role's abort) can never leave a warp blocked.
             if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;
             for (int rl = etid; rl < ng; rl += kEpiThreads) {
                 const int r = m * ng + rl;
-                if (r >= rows) break;
-                float4 acc4 = comb[rl];
+                float4 acc4 = stats[rl];
+                stats[rl] = kEmpty;
 #pragma unroll
-                for (int s4 = 1; s4 < 4; ++s4) acc4 = merge_stat(acc4, comb[s4 * kSwapMaxRows + rl]);
-                p.partials[static_cast<size_t>(r) * p.max_splits + 2 * g + static_cast<int>(rank)] = acc4;
+                for (int s4 = 1; s4 < 4; ++s4) {
+                    acc4 = merge_stat(acc4, stats[s4 * ng + rl]);
+                    stats[s4 * ng + rl] = kEmpty;
+                }
+                if (r < rows)
+                    p.partials[static_cast<size_t>(r) * p.max_splits + 2 * g + static_cast<int>(rank)] = acc4;
             }
             if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;
         }

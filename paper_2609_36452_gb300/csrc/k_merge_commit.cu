@@ -106,14 +106,16 @@ __global__ void __launch_bounds__(kBandThreads, 1) k_band(BandParams p) {
     }
     // 3. the second pass: the K-1 earlier window layers of the band positions
     const long long rows = static_cast<long long>(p.K - 1) * carry;
-    int mode, splits, swap_rows;
-    choose_head_tiling(rows, p.num_n_tiles, p.max_splits, p.pair_slots,
-                       p.hbm_tiles, p.tiling, mode, splits, swap_rows);
+    if (warp == 0) {
+        const HeadPlan hp = lookup_plan(rows, p.plan, p.plan_rows, p.plan_in);
+        if (lane == 0) {
+            p.meta[kMetaSwapRows] = hp.swap_rows;
+            p.meta[kMetaSplits] = hp.splits;
+            p.meta[kMetaHeadMode] = hp.mode;
+        }
+    }
     if (tid == 0) {
-        p.meta[kMetaSwapRows] = swap_rows;
         p.meta[kMetaRows] = static_cast<int>(rows);
-        p.meta[kMetaSplits] = splits;
-        p.meta[kMetaHeadMode] = mode;
         p.meta[kMetaSel] = carry;
         p.meta[kMetaLayer0] = 0;
         p.meta[kMetaRowsTotal] += static_cast<int>(rows);

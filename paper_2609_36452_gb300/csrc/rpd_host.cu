@@ -16,6 +16,7 @@
 #include <string>
 #include <vector>
 
+#include "head_plan.h"
 #include "rpd_internal.h"
 
 using namespace rpd;
@@ -112,6 +113,8 @@ struct rpd_ctx {
     int32_t *row_arg = nullptr;
     float *row_pmax = nullptr, *row_H = nullptr;
     int32_t *q_of_pos = nullptr, *pos_of_q = nullptr, *canvas_off = nullptr, *meta = nullptr;
+    HeadPlan *plan = nullptr;  // head-tiling plans by pass row count, rows 0..plan_rows
+    int plan_rows = 0;
     int32_t *sel_q = nullptr;  // lazy projection: compact indices of the band positions
     int32_t *band_off = nullptr;  // lazy projection: [B+1] each canvas's first band entry
     int projection = RPD_PROJECT_ALL;
@@ -136,7 +139,7 @@ struct rpd_ctx {
 
     void free_scratch() {
         void *ptrs[] = {u, inv_rms, partials, row_arg, row_pmax, row_H, q_of_pos, pos_of_q,
-                        canvas_off, meta, sel_q, band_off};
+                        canvas_off, meta, sel_q, band_off, plan};
         for (void *p : ptrs)
             if (p) cudaFree(p);
         u = nullptr;
@@ -145,11 +148,61 @@ struct rpd_ctx {
         row_arg = nullptr;
         row_pmax = row_H = nullptr;
         q_of_pos = pos_of_q = canvas_off = meta = sel_q = band_off = nullptr;
-        cap_bn = cap_b = cap_rows = 0;
+        plan = nullptr;
+        cap_bn = cap_b = cap_rows = plan_rows = 0;
     }
 };
 
 namespace {
+
+HeadPlanInputs plan_inputs(const rpd_ctx *c) {
+    HeadPlanInputs in;
+    in.num_n = (c->V + kTileN - 1) / kTileN;
+    in.max_splits = c->max_splits;
+    in.pair_slots = c->head_grid / 2;
+    in.hbm_tiles = head_stream_in_tiles(c->V, c->d, c->num_sms);
+    in.force = c->tiling;
+    return in;
+}
+
+// The head-tiling plan of every pass row count up to min(scratch rows, kPlanRows), evaluated
+// here (memoised by the quantities the plan depends on: the pair tile count, and the rows-on-N
+// group count and size) and uploaded to the device table the step's kernels look up.  The
+// stream must be idle (no step may be reading the table).
+int build_plan(rpd_ctx *c) {
+    const int n = std::min(c->cap_rows, kPlanRows);
+    if (!c->plan || n < 0) return RPD_OK;
+    const HeadPlanInputs in = plan_inputs(c);
+    const int gmax2 = std::min(in.num_n, in.max_splits);
+    const int gmax3 = std::min(in.num_n, in.max_splits / 2);
+    std::vector<HeadPlan> table(static_cast<size_t>(n) + 1);
+    std::vector<unsigned long long> key2((n + kPairTileM - 1) / kPairTileM + 1, 0ull);
+    std::vector<std::vector<unsigned long long>> key3;  // [groups][ng / step]
+    for (int r = 0; r <= n; ++r) {
+        if (r == 0 || in.pair_slots <= 0) {
+            table[r] = plan_head(r, in);
+            continue;
+        }
+        const int tiles2 = (r + kPairTileM - 1) / kPairTileM;
+        if (!key2[tiles2]) key2[tiles2] = best_split_key(kPairTileCost, tiles2, in.pair_slots, in.num_n, gmax2, 1, 1);
+        const int groups = swap_groups(r);
+        const int ng = swap_group_rows(r, groups);
+        unsigned long long k3 = ~0ull;
+        if (gmax3 > 0) {
+            if (static_cast<int>(key3.size()) <= groups) key3.resize(groups + 1);
+            std::vector<unsigned long long> &row = key3[groups];
+            const int slot = ng / kSwapRowStep;
+            if (static_cast<int>(row.size()) <= slot) row.resize(slot + 1, 0ull);
+            if (!row[slot]) row[slot] = best_split_key(swap_tile_cost(ng), groups, in.pair_slots, in.num_n, gmax3, 1, 1);
+            k3 = row[slot];
+        }
+        table[r] = plan_from_keys(in, key2[tiles2], k3, ng);
+    }
+    cudaError_t e = cudaMemcpy(c->plan, table.data(), table.size() * sizeof(HeadPlan), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(plan table)");
+    c->plan_rows = n;
+    return RPD_OK;
+}
 
 int ensure_scratch(rpd_ctx *c, int B, int N) {
     const long long bn = static_cast<long long>(B) * N;
@@ -182,6 +235,8 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
         {reinterpret_cast<void **>(&c->canvas_off), static_cast<size_t>(new_b + 1) * 4},
         {reinterpret_cast<void **>(&c->band_off), static_cast<size_t>(new_b + 1) * 4},
         {reinterpret_cast<void **>(&c->meta), kMetaWords * 4},
+        {reinterpret_cast<void **>(&c->plan),
+         (static_cast<size_t>(std::min<long long>(rows, kPlanRows)) + 1) * sizeof(HeadPlan)},
     };
     for (auto &a : allocs) {
         e = cudaMalloc(a.p, a.bytes);
@@ -204,6 +259,10 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
     for (int j = 0; rc == RPD_OK && j < kUMaps; ++j)
         rc = encode_bf16_2d(&c->maps.u_rows[j], c->u, static_cast<uint64_t>(rows), c->d,
                             static_cast<uint32_t>(kUBoxRows * (j + 1)));
+    if (rc == RPD_OK) {
+        e = cudaStreamSynchronize(c->stream);  // the memsets above precede the table upload
+        rc = e == cudaSuccess ? build_plan(c) : cuda_fail(e, "cudaStreamSynchronize");
+    }
     return rc;
 }
 
@@ -275,8 +334,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
 
     const int bn = B * N;
     const int num_n = (c->V + kTileN - 1) / kTileN;
-    const int pair_slots = c->head_grid / 2;
-    const float hbm_tiles = head_stream_in_tiles(c->V, c->d, c->num_sms);
+    const HeadPlanInputs plan_in = plan_inputs(c);
     // Lazy projection (forced, or chosen on the device per step): a second pass over the band.
     // It is not launched when even the largest possible row count keeps a single pass cheaper.
     const bool lazy = c->projection == RPD_PROJECT_LAZY ||
@@ -286,8 +344,8 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
     {
         KernelTimer t(c, 0);
         CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, B, N, c->K,
-                         num_n, c->max_splits, pair_slots, hbm_tiles, c->rule.block,
-                         c->projection == RPD_PROJECT_LAZY ? 1 : (lazy ? 2 : 0), c->tiling};
+                         plan_in, c->plan, c->plan_rows, c->rule.block,
+                         c->projection == RPD_PROJECT_LAZY ? 1 : (lazy ? 2 : 0)};
         e = launch_compact(cp, c->stream);
     }
     if (e != cudaSuccess) return cuda_fail(e, "compaction launch");
@@ -365,11 +423,9 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
             bp.N = N;
             bp.K = c->K;
             bp.theta_c = c->rule.theta_c;
-            bp.num_n_tiles = num_n;
-            bp.max_splits = c->max_splits;
-            bp.pair_slots = pair_slots;
-            bp.hbm_tiles = hbm_tiles;
-            bp.tiling = c->tiling;
+            bp.plan_in = plan_in;
+            bp.plan = c->plan;
+            bp.plan_rows = c->plan_rows;
             for (int b = 0; b < B; ++b) bp.tau[b] = tau[b];
             e = launch_band(bp, c->stream);
         }
@@ -508,8 +564,14 @@ int rpd_set_head_tiling(rpd_ctx *c, int tiling) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
     if (tiling < RPD_TILING_AUTO || tiling > RPD_TILING_ROWS_N)
         return fail(RPD_ERR_INVALID_ARGUMENT, "unknown head tiling %d", tiling);
+    if (tiling == c->tiling) return RPD_OK;
     c->tiling = tiling;
-    return RPD_OK;
+    if (!c->plan) return RPD_OK;
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
+    cudaError_t e = cudaStreamSynchronize(c->stream);  // no step may still read the plan table
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    return build_plan(c);
 }
 
 int rpd_set_wait_limit(rpd_ctx *c, int64_t microseconds) {

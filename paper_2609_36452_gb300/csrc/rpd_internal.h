@@ -29,22 +29,29 @@ constexpr int kPairStageBytesB = kPairHalfRows * kTileK * 2;
 // double-buffered in TMEM, a larger group uses all 512 columns once.
 constexpr int kSwapMaxRows = 512;
 constexpr int kSwapRowStep = 32;  // N of the M = 256 MMA: a multiple of 32, at least 32
-constexpr int kSwapMaxStages = 8;
+constexpr int kSwapMaxStages = 12;
 constexpr int kSwapStageBytesA = kPairHalfRows * kTileK * 2;
-constexpr int kSwapStageBudget = 192 * 1024;
-constexpr int kSwapEpiWarps = 8;
+
+constexpr int kSwapEpiWarps = 4;   // one per TMEM sub-partition, each taking all its chunks
 constexpr int kSwapXposeStride = 33;                             // floats per padded row
 constexpr int kSwapXposeBytes = kSwapEpiWarps * 32 * kSwapXposeStride * 4;  // 32 x 32 fp32 per warp
-static_assert(kSwapXposeBytes >= 4 * kSwapMaxRows * 16,
-              "the transpose blocks double as the [sub-partition][row] statistics exchange");
+// rows on N: running statistics [sub-partition][row of the group], 4 * ng float4
 constexpr int kUBoxRows = 16;  // granularity of a half group's rows (the TMA box heights)
-// Roles: warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-9 epilogue (pair tiles use warps 2-5).
+// Roles: warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-5 epilogue.  Six warps keep the kernel's
+// registers to about half of an SM's, so that the CTAs of the next kernel in the stream (launched
+// early, waiting on this grid) can already be resident when it finishes.
 constexpr int kHeadKernelThreads = 64 + 32 * kSwapEpiWarps;
 constexpr int kHeadBarrierBytes = 512;
-// The operand ring of either tiling, then the rows-on-N transpose blocks.
-constexpr int kHeadRegionBytes = kSwapStageBudget + kSwapXposeBytes;
+// The pair tiles' operand ring, or the rows-on-N ring, transpose blocks and statistics (the
+// ring takes what the other two leave).  The kernel keeps to about the pair ring's 192 KB: its
+// CTAs become resident (waiting) while the step's gather kernel still runs, and a larger
+// footprint leaves fewer gather CTAs room beside them (measured ~3 us a step at 211 KB).
+constexpr int kHeadRegionBytes = 193 * 1024;
 static_assert(kPairStages * (kPairStageBytesA + kPairStageBytesB) <= kHeadRegionBytes,
               "the pair tiles' operand ring fits the region");
+static_assert(kHeadRegionBytes - kSwapXposeBytes - 4 * kSwapMaxRows * 16 >=
+                  3 * (kSwapStageBytesA + (kSwapMaxRows / 2) * kTileK * 2),
+              "a 512-row group still gets three stages");
 // 1024-byte alignment slack + that region + barriers
 constexpr int kHeadKernelSmemBytes = 1024 + kHeadRegionBytes + kHeadBarrierBytes;
 static_assert(kHeadKernelSmemBytes <= 232448, "dynamic shared memory per CTA");
@@ -74,6 +81,24 @@ enum MetaIndex : int {
     kMetaWords = 16
 };
 
+// Tiling plan of a projection pass (head_plan.h): which tiling the head kernel runs, with how
+// many vocabulary splits.
+struct HeadPlan {
+    int mode;       // kHeadModePair or kHeadModeRowsN
+    int splits;     // partials per row the merge reads (vocabulary splits; twice that for rows on N)
+    int swap_rows;  // rows per group of the rows-on-N tiling (0 for pair tiles)
+    float est;      // estimated time, in 128 x 256-tile units
+};
+struct HeadPlanInputs {
+    int num_n;        // vocabulary tiles of 256
+    int max_splits;   // partials per row the scratch holds
+    int pair_slots;   // CTA pairs of the head kernel
+    float hbm_tiles;  // time to stream the head once, in tile units
+    int force;        // RPD_TILING_*
+};
+// Rows up to which a context tabulates the plan (larger passes evaluate it on the device).
+constexpr int kPlanRows = 16384;
+
 struct CompactParams {
     const uint8_t *mask;  // [B*N]
     int32_t *q_of_pos;    // [B*N] compact index or -1
@@ -81,13 +106,11 @@ struct CompactParams {
     int32_t *canvas_off;  // [B+1]
     int32_t *meta;        // [kMetaWords]
     int B, N, K;
-    int num_n_tiles;      // ceil(V / kTileN)
-    int max_splits;       // capacity of the partial-statistics buffer per row
-    int pair_slots;       // CTA pairs of the head kernel
-    float hbm_tiles;      // time to stream the head once, in pair-tile units (see below)
+    HeadPlanInputs plan_in;
+    const HeadPlan *plan; // [plan_rows + 1] plans by row count, or null
+    int plan_rows;
     int block;            // 0: every masked position; > 0: only each canvas's active block
     int lazy;             // 0: all window layers; 1: lazy; 2: lazy when it is estimated cheaper
-    int tiling;           // RPD_TILING_*: head tiling, or 0 to choose per pass
 };
 
 // Band fraction assumed when the device weighs lazy against full projection before the
@@ -116,21 +139,22 @@ struct BandParams {
     int32_t *band_off;         // out: [B+1] first band entry of each canvas
     int B, N, K;
     float theta_c;
-    int num_n_tiles, max_splits, pair_slots;
-    float hbm_tiles;
-    int tiling;
+    HeadPlanInputs plan_in;
+    const HeadPlan *plan;
+    int plan_rows;
     float tau[kMaxBatch];
 };
 
-// Costs of the tiling choice are in units of one 128-row x 256-entry tile's MMA work on one
-// SM.  A pair tile (256 rows on two SMs) costs kPairTileCost per SM: the measured per-SM rate
-// of the pair form on GB300 at the LLaDA head shape against that unit's nominal rate.
-constexpr float kPairTileCost = 0.88f;
-// "Rows on N" tiles: extra time of a group over 256 rows, whose epilogue cannot overlap the
-// next tile's MMAs (single-buffered TMEM), and the time per unit of operand bytes an SM
-// receives, relative to the 384 rows' worth of a 128 x 256 tile.
-constexpr float kSwapSingleBufferCost = 1.08f;
-constexpr float kSwapFeedCost = 1.0f;
+// Costs of the tiling choice are in units of one 128-row x 256-entry tile's MMA work on one SM
+// at the nominal rate below.  Both tilings are bound less by the MMAs than by how many operand
+// bytes an SM can keep in flight against the latency of its copies (a ring of ~192 KB against
+// ~2.5 us on GB300), so the per-tile costs are measured ones (LLaDA head, d = 4096, GB300):
+//   pair tile (256 rows x 256 entries per pair): 23.6 us, 0.97 units;
+//   rows-on-N tile (256 entries x a group of ng rows): about 0.80 + 0.0025 ng units, i.e.
+//   19.5 + 0.061 ng us (96 rows: 25 us, 288: 38 us, 448: 46 us, 512: 51 us).
+constexpr float kPairTileCost = 0.97f;
+constexpr float kSwapTileBase = 0.80f;
+constexpr float kSwapTilePerRow = 0.0025f;
 // Per-SM MMA rate of the unit tile and the sustained HBM read rate used by the tiling choice
 // (GB300 measurements; only their ratio matters).
 constexpr double kSingleTileFlopsPerSm = 1.1e13;

@@ -215,9 +215,12 @@ extern "C" int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, i
     // The per-step count/status words must start from zero on every call.
     cudaError_t e = cudaMemsetAsync(meta, 0, kMetaWords * 4, stream);
     if (e == cudaSuccess) {
-        CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, num_n, splits,
-                         pair_slots, head_stream_in_tiles(V, d, dev->num_sms),
-                         rule.block, 0, RPD_TILING_AUTO};
+        // no plan table (it would have to be allocated): the compaction kernel evaluates the
+        // head-tiling plan itself
+        const HeadPlanInputs plan_in{num_n, splits, pair_slots,
+                                     head_stream_in_tiles(V, d, dev->num_sms), RPD_TILING_AUTO};
+        CompactParams cp{mask, q_of_pos, pos_of_q, canvas_off, meta, 1, N, K, plan_in, nullptr, 0,
+                         rule.block, 0};
         e = launch_compact(cp, stream);
     }
     if (e == cudaSuccess) {
