@@ -692,6 +692,85 @@ def run_trajectory(args):
     print(json.dumps(out))
 
 
+def run_vocab_parallel(args):
+    """The LLaDA first step with the LM head split over the ranks (rank r holds slice r of the
+    vocabulary): per step every rank projects its slice, one NCCL all-gather moves 16 bytes per
+    projected row and rank, and every rank merges the slices and commits.  Strong scaling (the
+    same step on every N); at N = 1 the single slice is the whole head.  Timed like run_rpd."""
+    import torch.distributed as dist
+
+    import paper_2609_36452_gb300 as rpd
+    from paper_2609_36452_gb300.vocab_parallel import shard_bounds, sharded_step
+    rank, world, local = dist_env()
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+    os.environ.setdefault("MASTER_PORT", "29517")
+    dist.init_process_group("nccl", rank=rank, world_size=world, device_id=dev)
+    case = make_workload(0)  # every rank runs the same canvas
+    K, N, d, V = case["K"], case["N"], case["d"], case["V"]
+    v0, v1 = shard_bounds(V, world, rank)
+    W = case["W"][v0:v1].contiguous().to(dev)
+    g = case["g"].to(dev)
+    hidden = case["hidden"].to(dev).contiguous()
+    mask0 = case["mask"].to(dev)
+    ctx = rpd.Rpd(d, v1 - v0, K, case["eps"])
+    ctx.set_head(W, g)
+    ctx.set_vocab_shard(v0, V)
+    ctx.set_profile(case["rule"])
+    stream = torch.cuda.current_stream(dev)
+    ctx.set_stream(stream)
+    ctx.reserve(1, N)
+    n_masks = max(args.steps, args.warmup)
+    masks = mask0.unsqueeze(0).repeat(n_masks, 1).contiguous()
+    commit = torch.zeros(N, dtype=torch.uint8, device=dev)
+    token = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    stats = torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev)
+    partials = torch.empty(K, N, 4, dtype=torch.float32, device=dev)
+    gathered = torch.empty(world, K, N, 4, dtype=torch.float32, device=dev)
+
+    def steps(n):
+        for i in range(n):
+            sharded_step(ctx, hidden, masks[i % n_masks], case["tau"], case["budget"], commit, token,
+                         stats, partials=partials, gathered=gathered)
+
+    masks.copy_(mask0.unsqueeze(0).expand_as(masks))
+    steps(args.warmup)
+    torch.cuda.synchronize(dev)
+    assert rpd.stats_dict(stats.cpu())["status"] == 0
+    masks.copy_(mask0.unsqueeze(0).expand_as(masks))
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    steps(args.steps)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    dist.barrier()
+    t = torch.tensor([e0.elapsed_time(e1)], device=dev, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_step = float(t.item()) / args.steps
+    R = rows_of(case)
+    if rank == 0:
+        peaks = load_peaks()
+        roof = max(2.0 * R * d * V / (peaks["bf16_tflops"] * 1e12),
+                   (2.0 * V * d + 2.0 * R * d) / (peaks["hbm_gbs"] * 1e9))
+        print(json.dumps({
+            "metric": METRIC, "value": 1e3 / ms_step, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": dict(config_dict(case, R), workload="llada_first_step_vocab_parallel",
+                           parallelism=f"vocabulary slices over {world} GPUs, NCCL all-gather of "
+                                       f"{16 * R} bytes per rank and step"),
+            "rows_per_s": R * 1e3 / ms_step,
+            "step_roofline_frac_whole_job": roof / (ms_step * 1e-3) / world,
+            "gpu_launches": 7 * args.steps}))
+    ctx.close()
+    dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -710,6 +789,8 @@ def main():
                     help="head contraction tiling (default: chosen per pass on the device)")
     ap.add_argument("--cpu-positions", type=int, default=16,
                     help="positions of the oracle sample timed for cpu_baseline")
+    ap.add_argument("--vocab-parallel", action="store_true",
+                    help="LLaDA first step with the LM head split over the ranks (NCCL all-gather)")
     ap.add_argument("--no-trajectory", action="store_true",
                     help="leave the decode-trajectory object out of the default line")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -724,6 +805,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.vocab_parallel:
+        run_vocab_parallel(args)
     elif args.workload == "trajectory":
         run_trajectory(args)
     else:

@@ -207,6 +207,33 @@ int rpd_step_batched(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int B, int
 int rpd_step_host(rpd_ctx *ctx, const void *hidden, uint8_t *mask, int N, float tau,
                   float budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats);
 
+/* Vocabulary-parallel step over P devices (no counterpart in the paper: the same step as
+ * rpd_step, with the LM head's rows divided among devices).  Each device holds a contiguous
+ * slice of the head - rows [v_offset, v_offset + V) of a V_total-entry vocabulary, with V the
+ * context's vocabulary size - and runs, on the same hidden states and mask:
+ *   1. rpd_step_shard_partials: compaction, RMSNorm prologue and the head contraction over its
+ *      slice; writes, for every window layer k and masked position i, the softmax statistics
+ *      of the slice in base-2 units - (max, sum of 2^(x - max), sum of 2^(x - max)(x - max),
+ *      argmax as a global token index), x = logit * log2(e) - to out_partials[k][i] (float4,
+ *      [K][N][4] floats, device, 16-byte aligned; 16 bytes per projected row).  Entries of
+ *      positions that are not projected are left as they were.
+ *   2. the caller gathers every device's out_partials, in increasing v_offset order, into
+ *      [P][K][N][4] (one all-gather, e.g. NCCL), and
+ *   3. rpd_step_shard_finish: merges the P records of every projected row (in order; ties of
+ *      the argmax go to the lower token index, as in rpd_step), then scores, scans and commits
+ *      the canvas exactly as rpd_step does.  mask/out_* and tau/budget as in rpd_step; the mask
+ *      must be the one given to rpd_step_shard_partials, on the same context, with no other
+ *      step of the context in between.  out_stats->status reports this device's head waits.
+ * Every device then holds the same commits.  The projection must be RPD_PROJECT_ALL (lazy
+ * projection would need an exchange between its passes: RPD_ERR_UNSUPPORTED); RPD-block rules
+ * work unchanged.  rpd_set_vocab_shard: 0 <= v_offset and v_offset + V <= V_total. */
+int rpd_set_vocab_shard(rpd_ctx *ctx, int v_offset, int V_total);
+int rpd_step_shard_partials(rpd_ctx *ctx, const void *hidden, const uint8_t *mask, int N,
+                            float *out_partials);
+int rpd_step_shard_finish(rpd_ctx *ctx, const float *gathered, int P, uint8_t *mask, int N,
+                          float tau, float budget, uint8_t *out_commit, int32_t *out_token,
+                          rpd_stats *out_stats);
+
 /* Per-kernel timing with CUDA events recorded on the context's stream around every
  * launch while enabled.  rpd_kernel_times synchronises the recorded events and returns,
  * for each of the RPD_NUM_KERNELS kernels (gather/norm, head statistics, merge,

@@ -16,7 +16,8 @@ __all__ = [
     "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
     "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
-    "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_profile_enable", "rpd_kernel_times",
+    "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_set_vocab_shard",
+    "rpd_step_shard_partials", "rpd_step_shard_finish", "rpd_profile_enable", "rpd_kernel_times",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
 
@@ -101,6 +102,9 @@ def _load():
         "rpd_step_host": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_step_noalloc": (i32, [vp, vp, i32, i32, i32, f32, ctypes.POINTER(RpdRule), vp, vp,
                                    i32, f32, f32, vp, vp, vp, vp]),
+        "rpd_set_vocab_shard": (i32, [vp, i32, i32]),
+        "rpd_step_shard_partials": (i32, [vp, vp, vp, i32, vp]),
+        "rpd_step_shard_finish": (i32, [vp, vp, i32, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_profile_enable": (i32, [vp, i32]),
         "rpd_kernel_times": (i32, [vp, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_int64), i32]),
@@ -132,6 +136,9 @@ rpd_step = lib.rpd_step
 rpd_step_batched = lib.rpd_step_batched
 rpd_step_host = lib.rpd_step_host
 rpd_step_noalloc = lib.rpd_step_noalloc
+rpd_set_vocab_shard = lib.rpd_set_vocab_shard
+rpd_step_shard_partials = lib.rpd_step_shard_partials
+rpd_step_shard_finish = lib.rpd_step_shard_finish
 rpd_profile_enable = lib.rpd_profile_enable
 rpd_kernel_times = lib.rpd_kernel_times
 rpd_destroy = lib.rpd_destroy
@@ -291,6 +298,29 @@ class Rpd:
                 _arg(out_stats, "out_stats", "int32", STATS_WORDS, cuda=False))
         _check(rpd_step_host(self.handle, args[0], args[1], N, ctypes.c_float(tau),
                              ctypes.c_float(budget), *args[2:]))
+
+    def set_vocab_shard(self, v_offset: int, V_total: int):
+        """This context's head rows are vocabulary entries [v_offset, v_offset + V) of V_total."""
+        _check(rpd_set_vocab_shard(self.handle, int(v_offset), int(V_total)))
+
+    def step_shard_partials(self, hidden, mask, out_partials):
+        """Vocabulary-sharded step, part 1: hidden [K][N][d] bf16, mask [N] uint8 (read only),
+        out_partials [K][N][4] float32 (the slice's softmax statistics per projected row)."""
+        N = mask.numel()
+        args = (_arg(hidden, "hidden", "bfloat16", self.K * N * self.d), _arg(mask, "mask", "uint8"),
+                _arg(out_partials, "out_partials", "float32", self.K * N * 4))
+        _check(rpd_step_shard_partials(self.handle, args[0], args[1], N, args[2]))
+
+    def step_shard_finish(self, gathered, mask, tau, budget, out_commit, out_token, out_stats):
+        """Part 3: gathered [P][K][N][4] float32 (every slice's statistics, slices in vocabulary
+        order), then mask/out_* as in step()."""
+        N = mask.numel()
+        P = gathered.shape[0]
+        args = (_arg(gathered, "gathered", "float32", P * self.K * N * 4), _arg(mask, "mask", "uint8"),
+                _arg(out_commit, "out_commit", "uint8", N), _arg(out_token, "out_token", "int32", N),
+                _arg(out_stats, "out_stats", "int32", STATS_WORDS))
+        _check(rpd_step_shard_finish(self.handle, args[0], P, args[1], N, ctypes.c_float(tau),
+                                     ctypes.c_float(budget), *args[2:]))
 
     def profile(self, enable: bool):
         _check(rpd_profile_enable(self.handle, 1 if enable else 0))

@@ -114,7 +114,7 @@ __global__ void __maxnreg__(48) k_compact(CompactParams p) {
         p.meta[kMetaSwapRows] = swap_rows;
         p.meta[kMetaMasked] = carry;
         p.meta[kMetaRows] = static_cast<int>(rows);
-        p.meta[kMetaStatus] = RPD_OK;
+        if (!p.keep_status) p.meta[kMetaStatus] = RPD_OK;
         p.meta[kMetaSplits] = splits;
         p.meta[kMetaHeadMode] = mode;
         p.meta[kMetaSel] = carry;

@@ -45,6 +45,28 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge(MergeArgs mg, const int
     merge_pass_rows(mg, meta, sel_list, 0, meta[kMetaSel], blockIdx.x, gridDim.x);
 }
 
+// Merge of P vocabulary shards' statistics per (layer, masked position), shards in order.
+__global__ void __launch_bounds__(kMergeThreads) k_merge_shards(ShardMergeParams p) {
+    pdl_trigger();
+    pdl_wait();
+    const int nmt = p.meta[kMetaMasked];
+    const long long total = static_cast<long long>(p.K) * nmt;
+    for (long long r = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; r < total;
+         r += static_cast<long long>(gridDim.x) * blockDim.x) {
+        const int k = static_cast<int>(r / nmt);
+        const int q = static_cast<int>(r - static_cast<long long>(k) * nmt);
+        const int pos = p.pos_of_q[q];
+        Stat acc{-INFINITY, 0.f, 0.f, 0x7fffffff};
+        for (int sh = 0; sh < p.P; ++sh) {
+            const float4 v = p.gathered[(static_cast<size_t>(sh) * p.K + k) * p.BN + pos];
+            acc = merge2(acc, Stat{v.x, v.y, v.z, __float_as_int(v.w)});
+        }
+        p.row_arg[r] = acc.a;
+        p.row_pmax[r] = 1.0f / acc.s;
+        p.row_H[r] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
+    }
+}
+
 constexpr int kBandThreads = 1024;
 constexpr int kBandItems = 4;
 
@@ -445,6 +467,10 @@ cudaError_t launch_merge_score(const MergeArgs &mg, int32_t *meta, const int32_t
     if (items <= 2) return launch_pdl(k_merge_score<2>, g, t, 0, s, mg, meta, sel_list, p);
     if (items <= 4) return launch_pdl(k_merge_score<4>, g, t, 0, s, mg, meta, sel_list, p);
     return launch_pdl(k_merge_score<8>, g, t, 0, s, mg, meta, sel_list, p);
+}
+
+cudaError_t launch_merge_shards(const ShardMergeParams &p, int grid, cudaStream_t s) {
+    return launch_pdl(k_merge_shards, dim3(grid), dim3(kMergeThreads), 0, s, p);
 }
 
 cudaError_t launch_band(const BandParams &p, cudaStream_t s) {

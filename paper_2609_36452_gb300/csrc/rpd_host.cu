@@ -117,6 +117,8 @@ struct rpd_ctx {
     int plan_rows = 0;
     int32_t *sel_q = nullptr;  // lazy projection: compact indices of the band positions
     int32_t *band_off = nullptr;  // lazy projection: [B+1] each canvas's first band entry
+    int v_offset = 0, V_total = 0;  // vocabulary shard: rows of the head are entries
+                                    // [v_offset, v_offset + V) of a V_total vocabulary
     int projection = RPD_PROJECT_ALL;
     int tiling = RPD_TILING_AUTO;
     uint64_t wait_limit_ns = kWaitLimitNs;
@@ -307,6 +309,52 @@ int check_call(const rpd_ctx *c, float tau, float budget) {
     return RPD_OK;
 }
 
+ScoreParams score_params(const rpd_ctx *c, uint8_t *mask, int B, int N, const float *tau,
+                         const float *budget, uint8_t *out_commit, int32_t *out_token,
+                         rpd_stats *out_stats, bool lazy) {
+    ScoreParams sp{};
+    sp.mask = mask;
+    sp.q_of_pos = c->q_of_pos;
+    sp.canvas_off = c->canvas_off;
+    sp.meta = c->meta;
+    sp.row_arg = c->row_arg;
+    sp.row_pmax = c->row_pmax;
+    sp.row_H = c->row_H;
+    sp.out_commit = out_commit;
+    sp.out_token = out_token;
+    sp.out_stats = out_stats;
+    sp.dbg = c->dbg;
+    sp.B = B;
+    sp.N = N;
+    sp.K = c->K;
+    sp.theta_c = c->rule.theta_c;
+    sp.theta_s = c->rule.theta_s;
+    sp.w = c->rule.w;
+    sp.k_max = c->rule.k_max;
+    sp.window = c->rule.window;
+    sp.block = c->rule.block;
+    sp.lazy = lazy ? 1 : 0;
+    for (int b = 0; b < B; ++b) {
+        sp.tau[b] = tau[b];
+        sp.budget[b] = budget[b];
+    }
+    return sp;
+}
+
+// Arguments every single-canvas step checks before it touches the GPU.
+int check_canvas(const rpd_ctx *c, const void *hidden, const void *mask, int N) {
+    if (!c->W || !c->g) return fail(RPD_ERR_NO_HEAD, "rpd_set_head has not been called");
+    if (N < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be >= 0");
+    if (N > kMaxCanvas) return fail(RPD_ERR_UNSUPPORTED, "N must be <= %d", kMaxCanvas);
+    if (N > 0 && (!hidden || !mask)) return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
+    if (hidden && !aligned16(hidden))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "hidden must be 16-byte aligned");
+    if (hidden && !pointer_usable(hidden, c->device, true))
+        return fail(RPD_ERR_INVALID_ARGUMENT,
+                    "hidden must be device memory of the context's device or mapped page-locked host memory");
+    return RPD_OK;
+}
+
 int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const float *tau,
              const float *budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats) {
     if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
@@ -351,32 +399,8 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
     if (e != cudaSuccess) return cuda_fail(e, "compaction launch");
 
     // Scoring, scan and commit of every canvas (k_score_commit, or the last merge's grid).
-    ScoreParams sp{};
-    sp.mask = mask;
-    sp.q_of_pos = c->q_of_pos;
-    sp.canvas_off = c->canvas_off;
-    sp.meta = c->meta;
-    sp.row_arg = c->row_arg;
-    sp.row_pmax = c->row_pmax;
-    sp.row_H = c->row_H;
-    sp.out_commit = out_commit;
-    sp.out_token = out_token;
-    sp.out_stats = out_stats;
-    sp.dbg = c->dbg;
-    sp.B = B;
-    sp.N = N;
-    sp.K = c->K;
-    sp.theta_c = c->rule.theta_c;
-    sp.theta_s = c->rule.theta_s;
-    sp.w = c->rule.w;
-    sp.k_max = c->rule.k_max;
-    sp.window = c->rule.window;
-    sp.block = c->rule.block;
-    sp.lazy = lazy ? 1 : 0;
-    for (int b = 0; b < B; ++b) {
-        sp.tau[b] = tau[b];
-        sp.budget[b] = budget[b];
-    }
+    const ScoreParams sp = score_params(c, mask, B, N, tau, budget, out_commit, out_token,
+                                        out_stats, lazy);
     const bool fuse_score = B == 1 && N <= kFuseScoreMaxN;
 
     // One projection pass: gather + RMSNorm prologue, head statistics, merge.  Rows, layers
@@ -675,6 +699,95 @@ int rpd_step_host(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float ta
     std::memcpy(out_commit, h + (off_commit - off_mask), static_cast<size_t>(N));
     std::memcpy(out_token, h + (off_token - off_mask), static_cast<size_t>(N) * 4);
     std::memcpy(out_stats, h + (off_stats - off_mask), sizeof(rpd_stats));
+    return RPD_OK;
+}
+
+int rpd_set_vocab_shard(rpd_ctx *c, int v_offset, int V_total) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (v_offset < 0 || V_total < c->V || v_offset > V_total - c->V)
+        return fail(RPD_ERR_INVALID_ARGUMENT,
+                    "shard [%d, %d + %d) must lie inside a vocabulary of %d entries", v_offset,
+                    v_offset, c->V, V_total);
+    c->v_offset = v_offset;
+    c->V_total = V_total;
+    return RPD_OK;
+}
+
+int rpd_step_shard_partials(rpd_ctx *c, const void *hidden, const uint8_t *mask, int N,
+                            float *out_partials) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
+    int rc = check_canvas(c, hidden, mask, N);
+    if (rc) return rc;
+    if (c->projection != RPD_PROJECT_ALL)
+        return fail(RPD_ERR_UNSUPPORTED,
+                    "vocabulary-sharded steps project every window layer (RPD_PROJECT_ALL)");
+    if (N == 0) return RPD_OK;
+    if (!out_partials || !aligned16(out_partials))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "out_partials must be 16-byte aligned device memory");
+    rc = ensure_scratch(c, 1, N);
+    if (rc) return rc;
+    const HeadPlanInputs plan_in = plan_inputs(c);
+    CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, 1, N, c->K,
+                     plan_in, c->plan, c->plan_rows, c->rule.block, 0};
+    cudaError_t e = launch_compact(cp, c->stream);
+    if (e == cudaSuccess) {
+        NormParams np{static_cast<const __nv_bfloat16 *>(hidden),
+                      static_cast<const __nv_bfloat16 *>(c->g), c->pos_of_q, nullptr, c->meta,
+                      c->u, c->inv_rms, N, c->d, c->eps};
+        const long long max_rows = static_cast<long long>(c->K) * N;
+        e = launch_gather_norm(np, static_cast<int>(std::min<long long>(c->num_sms * 8, (max_rows + 7) / 8)),
+                               c->stream);
+    }
+    if (e == cudaSuccess) {
+        HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits, c->wait_limit_ns,
+                      c->stall_next ? 1 : 0};
+        e = launch_head(c->maps, hp, c->head_grid, c->stream);
+        c->stall_next = false;
+    }
+    if (e == cudaSuccess) {
+        MergeArgs mg{c->partials, c->max_splits, c->row_arg, c->row_pmax, c->row_H,
+                     reinterpret_cast<float4 *>(out_partials), c->pos_of_q, N, c->v_offset};
+        e = launch_merge(mg, c->meta, nullptr, c->num_sms * 4, c->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "sharded projection launch");
+    return RPD_OK;
+}
+
+int rpd_step_shard_finish(rpd_ctx *c, const float *gathered, int P, uint8_t *mask, int N, float tau,
+                          float budget, uint8_t *out_commit, int32_t *out_token,
+                          rpd_stats *out_stats) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
+    if (P < 1 || P > 4096) return fail(RPD_ERR_INVALID_ARGUMENT, "P must be in [1, 4096]");
+    int rc = check_call(c, tau, budget);
+    if (rc) return rc;
+    if (N < 0) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be >= 0");
+    if (N > kMaxCanvas) return fail(RPD_ERR_UNSUPPORTED, "N must be <= %d", kMaxCanvas);
+    if (N == 0) return RPD_OK;
+    if (!gathered || !mask || !out_commit || !out_token || !out_stats)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "null buffer");
+    if (!aligned16(gathered)) return fail(RPD_ERR_INVALID_ARGUMENT, "gathered must be 16-byte aligned");
+    rc = ensure_scratch(c, 1, N);
+    if (rc) return rc;
+    const HeadPlanInputs plan_in = plan_inputs(c);
+    CompactParams cp{mask, c->q_of_pos, c->pos_of_q, c->canvas_off, c->meta, 1, N, c->K,
+                     plan_in, c->plan, c->plan_rows, c->rule.block, 0,
+                     1 /* keep the partials call's status (a timed-out wait) */};
+    cudaError_t e = launch_compact(cp, c->stream);
+    if (e == cudaSuccess) {
+        ShardMergeParams mp{reinterpret_cast<const float4 *>(gathered), P, c->K, N, c->pos_of_q,
+                            c->meta, c->row_arg, c->row_pmax, c->row_H};
+        e = launch_merge_shards(mp, c->num_sms * 2, c->stream);
+    }
+    if (e == cudaSuccess) {
+        const ScoreParams sp = score_params(c, mask, 1, N, &tau, &budget, out_commit, out_token,
+                                            out_stats, false);
+        e = launch_score_commit(sp, c->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "shard merge / score launch");
     return RPD_OK;
 }
 

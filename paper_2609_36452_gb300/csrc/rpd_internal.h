@@ -111,6 +111,7 @@ struct CompactParams {
     int plan_rows;
     int block;            // 0: every masked position; > 0: only each canvas's active block
     int lazy;             // 0: all window layers; 1: lazy; 2: lazy when it is estimated cheaper
+    int keep_status;      // 1: leave the status word as the previous call of the step left it
 };
 
 // Band fraction assumed when the device weighs lazy against full projection before the
@@ -125,6 +126,26 @@ constexpr float kLazyBandGuess = 0.25f;
 struct MergeArgs {
     const float4 *partials;  // [rows][max_splits]
     int max_splits;
+    int32_t *row_arg;
+    float *row_pmax;
+    float *row_H;
+    // Vocabulary-sharded steps: when shard_out is set, each row's merged statistics themselves
+    // (max, sum, tsum, argmax + v_offset) go to shard_out[layer * shard_stride + position]
+    // instead of the derived outputs above.
+    float4 *shard_out;
+    const int32_t *pos_of_q;
+    int shard_stride;
+    int v_offset;
+};
+
+// Merge of the statistics of P vocabulary shards (rpd_step_shard_finish): per (layer k, masked
+// position) the P records gathered[(p * K + k) * N + position], p = 0..P-1 in order, give the
+// row's argmax, probability and entropy at k * NMT + q.
+struct ShardMergeParams {
+    const float4 *gathered;   // [P][K][B*N]
+    int P, K, BN;
+    const int32_t *pos_of_q;  // [NMT]
+    const int32_t *meta;
     int32_t *row_arg;
     float *row_pmax;
     float *row_H;
@@ -150,11 +171,11 @@ struct BandParams {
 // bytes an SM can keep in flight against the latency of its copies (a ring of ~192 KB against
 // ~2.5 us on GB300), so the per-tile costs are measured ones (LLaDA head, d = 4096, GB300):
 //   pair tile (256 rows x 256 entries per pair): 23.6 us, 0.97 units;
-//   rows-on-N tile (256 entries x a group of ng rows): about 0.80 + 0.0025 ng units, i.e.
-//   19.5 + 0.061 ng us (96 rows: 25 us, 288: 38 us, 448: 46 us, 512: 51 us).
+//   rows-on-N tile (256 entries x a group of ng rows): about 0.80 + 0.0027 ng units, i.e.
+//   19.5 + 0.066 ng us (96 rows: 25 us, 288: 38 us, 384: 46 us, 448: 46 us, 512: 51 us).
 constexpr float kPairTileCost = 0.97f;
 constexpr float kSwapTileBase = 0.80f;
-constexpr float kSwapTilePerRow = 0.0025f;
+constexpr float kSwapTilePerRow = 0.0027f;
 // Per-SM MMA rate of the unit tile and the sustained HBM read rate used by the tiling choice
 // (GB300 measurements; only their ratio matters).
 constexpr double kSingleTileFlopsPerSm = 1.1e13;
@@ -297,6 +318,7 @@ cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t
                          int grid, cudaStream_t s);
 cudaError_t launch_band(const BandParams &p, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
+cudaError_t launch_merge_shards(const ShardMergeParams &p, int grid, cudaStream_t s);
 // The step's last merge fused with the scoring of its canvas (one canvas of at most
 // kFuseScoreMaxN positions); the separate score launch is then skipped.
 constexpr int kFuseScoreMaxN = 2048;

@@ -95,10 +95,16 @@ __device__ int merge_pass_rows(const MergeArgs &mg, const int32_t *meta, const i
             acc = (gl & o) ? merge2(other, acc) : merge2(acc, other);  // fixed operand order
         }
         if (valid && gl == 0) {
-            const size_t out = static_cast<size_t>(layer0 + kr) * nmt + (sel_list ? sel_list[s] : s);
-            mg.row_arg[out] = acc.a;
-            mg.row_pmax[out] = 1.0f / acc.s;
-            mg.row_H[out] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
+            const int q = sel_list ? sel_list[s] : s;
+            if (mg.shard_out) {
+                mg.shard_out[static_cast<size_t>(layer0 + kr) * mg.shard_stride + mg.pos_of_q[q]] =
+                    make_float4(acc.m, acc.s, acc.t, __int_as_float(acc.a + mg.v_offset));
+            } else {
+                const size_t out = static_cast<size_t>(layer0 + kr) * nmt + q;
+                mg.row_arg[out] = acc.a;
+                mg.row_pmax[out] = 1.0f / acc.s;
+                mg.row_H[out] = fmaxf(logf(acc.s) - kLn2 * (acc.t / acc.s), 0.f);
+            }
         }
     }
     return min(cta_slots, (total + groups - 1) / groups);
