@@ -38,12 +38,10 @@ UNIT = "commit-steps/s"
 # DRAM bytes (read + write) per head-statistics launch from ncu captures, keyed by workload
 # and by a hash of the kernel's sources at capture time; any source change makes it null.
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
-                "paper_2609_36452_gb300/csrc/rpd_internal.h")
+                "paper_2609_36452_gb300/csrc/rpd_internal.h", "paper_2609_36452_gb300/csrc/head_plan.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "2bf1e6957f760dfb"): 1.0494e9,
-    ("llada_tail_5_masked", "2bf1e6957f760dfb"): 1.0437e9,
-    ("batched_serving", "2bf1e6957f760dfb"): 8.822e9,
-    ("dream_mid_decode", "2bf1e6957f760dfb"): 1.1033e9,
+    ("llada_first_step", "c607d0d4a3e65b8d"): 1.0512e9,
+    ("llada_tail_70_masked", "c607d0d4a3e65b8d"): 1.0558e9,
 }
 
 # Nominal dense rates of GB300 (context only; the fractions use the measured peaks).
