@@ -269,6 +269,7 @@ def config_dict(case, R):
             "projection": "lazy" if "lazy_rows" in case else "all window layers",
             "rows_projected": case.get("lazy_rows", R),
             "head_tiling": case.get("tiling", "auto (per pass, on the device)"),
+            "head_layout": case.get("head_layout", "tiled (context copy of W in contiguous 128 x 64 blocks)"),
             "l2": f"inputs larger than L2: the {2 * case['V'] * case['d'] / 1e9:.2f} GB head is streamed every step"}
 
 
@@ -339,15 +340,19 @@ def run_rpd(args):
     stats = torch.zeros(B, rpd.STATS_WORDS, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     ctx = rpd.Rpd(d, V, K, case["eps"])
+    ctx.set_stream(stream)
+    ctx.set_head_layout(args.head_layout)
     ctx.set_head(W, g)
     ctx.set_profile(case["rule"])
-    ctx.set_stream(stream)
     ctx.reserve(B, N)
     ctx.set_projection(args.projection)
     ctx.set_head_tiling(args.tiling)
     if args.tiling != "auto":
         case["name"] = case["name"] + "_" + args.tiling
         case["tiling"] = args.tiling
+    if args.head_layout != "tiled":
+        case["name"] = case["name"] + "_" + args.head_layout
+        case["head_layout"] = "borrowed (W read in place, row-major)"
 
     def refill_masks():
         masks.copy_(mask0.unsqueeze(0).expand_as(masks))
@@ -783,6 +788,9 @@ def main():
     ap.add_argument("--projection", choices=["all", "lazy", "auto"], default="all",
                     help="window layers projected: all (the step as defined), lazy (earlier "
                          "layers only for band positions), auto (chosen per step on the device)")
+    ap.add_argument("--head-layout", choices=["tiled", "borrowed"], default="tiled",
+                    help="how the head kernel reads W: the context's tiled copy (default) or the "
+                         "caller's row-major tensor in place")
     ap.add_argument("--tiling", choices=["auto", "pair", "rows_n"], default="auto",
                     help="head contraction tiling (default: chosen per pass on the device)")
     ap.add_argument("--cpu-positions", type=int, default=16,

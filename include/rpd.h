@@ -102,12 +102,30 @@ typedef struct rpd_debug {
  * Returns NULL on failure (see rpd_last_error()). */
 rpd_ctx *rpd_create(int d, int V, int K, float eps);
 
-/* Borrow the LM head W_head ([V][d] bf16, row v = token v's output embedding, device,
- * 16-byte aligned) and the final-norm gain g_norm ([d] bf16, device, 16-byte aligned).
- * Both must stay valid until the context is destroyed or the head is replaced; the
- * library keeps no copy.  Host memory, or memory of another device, is refused with
- * RPD_ERR_INVALID_ARGUMENT.  App. A.2: the model's own final normalisation and head. */
+/* Set the LM head W_head ([V][d] bf16, row v = token v's output embedding, device, 16-byte
+ * aligned) and the final-norm gain g_norm ([d] bf16, device, 16-byte aligned).  g_norm is
+ * borrowed: it must stay valid until the context is destroyed or the head is replaced.
+ * W_head is copied into the context's tiled layout and not read after the call returns, or
+ * borrowed in the same way as g_norm (see rpd_set_head_layout).  The copy runs on the
+ * context's stream and the call waits for it.  Host memory, or memory of another device, is
+ * refused with RPD_ERR_INVALID_ARGUMENT.  App. A.2: the model's own final normalisation and
+ * head. */
 int rpd_set_head(rpd_ctx *ctx, const void *W_head, const void *g_norm);
+
+/* Layout in which the head kernel reads W (no counterpart in the paper; the results are
+ * bitwise the same in both).
+ *   RPD_HEAD_TILED (default): rpd_set_head copies W into context-owned device memory as
+ *     contiguous blocks of 128 rows x 64 columns (16 KB; block (t, k) holds rows
+ *     [128t, 128t + 128) and columns [64k, 64k + 64), blocks ordered by t, then k, rows past V
+ *     zero), so that every block the head kernel stages is one contiguous read.  It costs
+ *     ceil(V/128)*128*d*2 bytes of device memory (1.04 GB at the LLaDA-8B head) and one copy
+ *     per rpd_set_head.  Needs d % 64 == 0; with other d the context borrows W_head.
+ *   RPD_HEAD_BORROWED: the head kernel reads W_head in place; W_head must stay valid like
+ *     g_norm, and nothing is copied.
+ * Takes effect at the next rpd_set_head.  Other values: RPD_ERR_INVALID_ARGUMENT. */
+#define RPD_HEAD_TILED 0
+#define RPD_HEAD_BORROWED 1
+int rpd_set_head_layout(rpd_ctx *ctx, int layout);
 
 /* Replace the rule parameters (Table 4).  Requires 0 <= theta_c, w >= 0, k_max >= 1,
  * window >= 1, block >= 0.  theta_c < tau is checked per step (Eq. 5 requires theta_c < theta_h). */
@@ -274,7 +292,8 @@ int rpd_step_noalloc(const void *W_head, const void *g_norm, int d, int V, int K
                      float budget, uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats,
                      void *stream);
 
-/* Free the context and its scratch (not the borrowed head).  NULL is ignored. */
+/* Free the context, its scratch and its copy of the head (not the caller's buffers).  NULL
+ * is ignored. */
 void rpd_destroy(rpd_ctx *ctx);
 
 /* Message of the last failing call on this host thread ("" if none). */

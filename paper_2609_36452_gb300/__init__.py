@@ -15,7 +15,7 @@ __all__ = [
     "RPD_OK", "RPD_ERR_INVALID_ARGUMENT", "RPD_ERR_NO_HEAD", "RPD_ERR_CUDA",
     "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
-    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
+    "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_head_layout", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_set_vocab_shard",
     "rpd_step_shard_partials", "rpd_step_shard_finish", "rpd_profile_enable", "rpd_kernel_times",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
@@ -70,6 +70,9 @@ RPD_TILING_AUTO = 0
 RPD_TILING_PAIR = 1
 RPD_TILING_ROWS_N = 2
 HEAD_TILINGS = {"auto": RPD_TILING_AUTO, "pair": RPD_TILING_PAIR, "rows_n": RPD_TILING_ROWS_N}
+RPD_HEAD_TILED = 0
+RPD_HEAD_BORROWED = 1
+HEAD_LAYOUTS = {"tiled": RPD_HEAD_TILED, "borrowed": RPD_HEAD_BORROWED}
 
 
 class RpdError(RuntimeError):
@@ -95,6 +98,7 @@ def _load():
         "rpd_set_debug": (i32, [vp, ctypes.POINTER(RpdDebug)]),
         "rpd_set_projection": (i32, [vp, i32]),
         "rpd_set_head_tiling": (i32, [vp, i32]),
+        "rpd_set_head_layout": (i32, [vp, i32]),
         "rpd_set_wait_limit": (i32, [vp, ctypes.c_int64]),
         "rpd_inject_stall": (i32, [vp]),
         "rpd_step": (i32, [vp, vp, vp, i32, f32, f32, vp, vp, vp]),
@@ -130,6 +134,7 @@ rpd_reserve = lib.rpd_reserve
 rpd_set_debug = lib.rpd_set_debug
 rpd_set_projection = lib.rpd_set_projection
 rpd_set_head_tiling = lib.rpd_set_head_tiling
+rpd_set_head_layout = lib.rpd_set_head_layout
 rpd_set_wait_limit = lib.rpd_set_wait_limit
 rpd_inject_stall = lib.rpd_inject_stall
 rpd_step = lib.rpd_step
@@ -179,7 +184,8 @@ _DEBUG_DTYPES = {"conf": "float32", "entropy": "float32", "persist": "int32", "d
 
 class Rpd:
     """A context bound to torch tensors.  ``W`` ([V][d]) and ``g`` ([d]) are bf16 CUDA
-    tensors that must outlive the context (the library borrows them)."""
+    tensors; this object keeps references to both, so they outlive the context (the library
+    borrows ``g``, and ``W`` too under the "borrowed" head layout)."""
 
     def __init__(self, d: int, V: int, K: int, eps: float = 1e-6):
         self.d, self.V, self.K, self.eps = d, V, K, eps
@@ -230,6 +236,12 @@ class Rpd:
         if isinstance(mode, bool):
             mode = "lazy" if mode else "all"
         _check(rpd_set_projection(self.handle, PROJECTION_MODES[mode]))
+
+    def set_head_layout(self, layout):
+        """How the head kernel reads W: "tiled" (default: set_head copies W into contiguous
+        128 x 64 blocks owned by the context) or "borrowed" (W read in place, kept alive by
+        this object).  Takes effect at the next set_head."""
+        _check(rpd_set_head_layout(self.handle, HEAD_LAYOUTS[layout]))
 
     def set_head_tiling(self, tiling):
         """Tiling of the head contraction: "auto" (default, chosen per pass on the device),

@@ -21,8 +21,9 @@
 //                padded to a multiple of 32), so that a pass whose row count is not a multiple
 //                of 256 pads by at most 31 rows per group.
 // Roles: warp 0 TMA producer (one thread), warp 1 TMEM owner (512 columns) and MMA issuer
-// (one thread, even CTA), warps 2-5 epilogue.  Every wait is bounded; a
-// timeout latches RPD_ERR_TIMEOUT in the step's status word and the CTA drains and exits.
+// (one thread, even CTA), warps 2-9 epilogue (pair tiles use warps 2-5).  Every wait is
+// bounded; a timeout latches RPD_ERR_TIMEOUT in the step's status word and the CTA drains and
+// exits.
 #include <atomic>
 
 #include "ptx.cuh"
@@ -277,8 +278,12 @@ __device__ __forceinline__ void head_pair(const CUtensorMap *tmU, const CUtensor
                         uint8_t *st = sm.ring + stage * kStageBytes;
                         tma_load_2d_pair(st, tmU, fb, kb * kTileK,
                                          m * kPairTileM + static_cast<int>(rank) * kPairHalfRows);
-                        tma_load_2d_pair(st + kPairStageBytesA, tmW, fb, kb * kTileK,
-                                         n * kTileN + static_cast<int>(rank) * kPairHalfRows);
+                        if (p.w_tiled)  // block (2n + rank, kb): 128 contiguous rows of 64
+                            tma_load_2d_pair(st + kPairStageBytesA, tmW, fb, 0,
+                                             ((2 * n + static_cast<int>(rank)) * num_kb + kb) * kPairHalfRows);
+                        else
+                            tma_load_2d_pair(st + kPairStageBytesA, tmW, fb, kb * kTileK,
+                                             n * kTileN + static_cast<int>(rank) * kPairHalfRows);
                         ++fills;
                         if (++stage == kPairStages) {
                             stage = 0;
@@ -558,7 +563,11 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                         const uint32_t fb = full0 + static_cast<uint32_t>(stage * sizeof(uint64_t));
                         uint8_t *st = sm.ring + stage * stage_bytes;
                         const int x = kb * kTileK;
-                        tma_load_2d_pair(st, tmW, fb, x, n * kTileN + w_off);
+                        if (p.w_tiled)  // block (2n + rank, kb): 128 contiguous rows of 64
+                            tma_load_2d_pair(st, tmW, fb, 0,
+                                             ((2 * n + static_cast<int>(rank)) * num_kb + kb) * kPairHalfRows);
+                        else
+                            tma_load_2d_pair(st, tmW, fb, x, n * kTileN + w_off);
                         uint8_t *sb = st + kSwapStageBytesA;
                         tma_load_2d_pair(sb, map0, fb, x, rows0);
                         if (half1 > 0) tma_load_2d_pair(sb + half0 * (kTileK * 2), map1, fb, x, rows1);
@@ -640,8 +649,10 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
         }
     } else {
         // ---------------------------------------------------------- epilogue (both CTAs)
-        const int sub = warp & 3;                // TMEM sub-partition (lanes 32*sub..+31)
-        const int etid = (warp - 2) * 32 + lane; // 0 .. kEpiThreads-1
+        const int sub = warp & 3;                 // TMEM sub-partition (lanes 32*sub..+31)
+        const int etid = (warp - 2) * 32 + lane;  // 0 .. kEpiThreads-1
+        const int chunk0 = (warp - 2) / 4;        // the two warps of a sub-partition alternate chunks
+        constexpr int kChunkStep = kSwapEpiWarps / 4;
         const int nch = ng / 32;
         const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
         const uint32_t acc_empty0 = mapa_shared(smem_u32(&acc_empty[0]), 0);
@@ -676,7 +687,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                 const int vbase = n * kTileN + static_cast<int>(rank) * kPairHalfRows + sub * 32;
                 const bool full_tile = vbase + 32 <= p.V;
 #pragma unroll 1
-                for (int c = 0; c < nch; ++c) {
+                for (int c = chunk0; c < nch; c += kChunkStep) {
                     float v[32];
                     tmem_ld_32x32b_x32(lane_base + acc * kTileN + c * 32, v);
                     // thread `lane` holds vocabulary entry vbase + lane for rows c*32 + i; write
@@ -756,6 +767,25 @@ __global__ void __launch_bounds__(kHeadKernelThreads, 1)
         head_swap(maps.u_rows, &maps.w128, p, sm, rows, splits / 2, p.meta[kMetaSwapRows]);
 }
 
+// The tiled copy of the head: thread i writes 16-byte vector i of Wt, which is vector k8 of
+// row r of block blk = t * (d / 64) + k, i.e. W[128 t + r][64 k + 8 k8 ...].
+__global__ void k_tile_head(const uint4 *__restrict__ W, uint4 *__restrict__ Wt, int V, int d) {
+    const int nkb = d / 64;
+    const long long total = static_cast<long long>((V + 127) / 128) * nkb * 128 * 8;
+    for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<long long>(gridDim.x) * blockDim.x) {
+        const int k8 = static_cast<int>(i & 7);
+        const long long rest = i >> 3;
+        const int r = static_cast<int>(rest & 127);
+        const long long blk = rest >> 7;
+        const int k = static_cast<int>(blk % nkb);
+        const int row = static_cast<int>(blk / nkb) * 128 + r;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (row < V) v = W[(static_cast<long long>(row) * d + k * 64) / 8 + k8];
+        Wt[i] = v;
+    }
+}
+
 // Per-device one-time settings (the dynamic shared-memory opt-in is a property of the
 // kernel on each device).
 constexpr int kMaxDevices = 64;
@@ -801,6 +831,11 @@ int head_max_clusters() {
     if (cudaOccupancyMaxActiveClusters(&n, k_head, &cfg) != cudaSuccess) n = 0;
     g_head_clusters[dev].store(n + 1, std::memory_order_release);
     return n;
+}
+
+cudaError_t launch_tile_head(const void *W, void *Wt, int V, int d, cudaStream_t s) {
+    k_tile_head<<<1024, 256, 0, s>>>(static_cast<const uint4 *>(W), static_cast<uint4 *>(Wt), V, d);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_head(const HeadMaps &maps, const HeadParams &p, int grid, cudaStream_t s) {

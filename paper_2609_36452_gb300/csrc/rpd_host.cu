@@ -101,6 +101,8 @@ struct rpd_ctx {
     float eps = 0.f;
     int device = 0, num_sms = 0;
     const void *W = nullptr, *g = nullptr;
+    int head_layout = RPD_HEAD_TILED;
+    void *W_tiled = nullptr;  // the tiled copy of the head (RPD_HEAD_TILED), else null
     rpd_rule rule{0.6f, 3.5f, 15.0f, 6, 32, 0};
     cudaStream_t stream = nullptr;
     rpd_debug dbg{};
@@ -422,7 +424,7 @@ int run_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const 
         {
             KernelTimer t(c, 1);
             HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits,
-                          c->wait_limit_ns, c->stall_next ? 1 : 0};
+                          c->wait_limit_ns, c->stall_next ? 1 : 0, c->W_tiled != nullptr ? 1 : 0};
             // One launch: the kernel reads the tiling chosen on the device for this pass.
             err = launch_head(c->maps, hp, c->head_grid, c->stream);
         }
@@ -537,9 +539,37 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
     if (!pointer_usable(W_head, c->device, false) || !pointer_usable(g_norm, c->device, false))
         return fail(RPD_ERR_INVALID_ARGUMENT,
                     "W_head and g_norm must be device memory on the context's device");
+    // No step may still read the previous head (or its tiled copy) once it is replaced.
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    if (c->W_tiled) cudaFree(c->W_tiled);
+    c->W_tiled = nullptr;
+    c->W = nullptr;
     CUtensorMap m2;
-    int rc = encode_bf16_2d(&m2, W_head, static_cast<uint64_t>(c->V), c->d, kPairHalfRows);
-    if (rc) return rc;
+    int rc;
+    if (c->head_layout == RPD_HEAD_TILED && c->d % 64 == 0) {
+        // rows as 2-D tensor map rows of 64 columns: block (t, k) is map rows
+        // [128 (t (d/64) + k), +128)
+        const uint64_t vpad = (static_cast<uint64_t>(c->V) + 127) / 128 * 128;
+        void *wt = nullptr;
+        e = cudaMalloc(&wt, vpad * static_cast<uint64_t>(c->d) * 2);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(tiled head)");
+        e = launch_tile_head(W_head, wt, c->V, c->d, c->stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+        if (e != cudaSuccess) {
+            cudaFree(wt);
+            return cuda_fail(e, "tiled copy of the head");
+        }
+        rc = encode_bf16_2d(&m2, wt, vpad * static_cast<uint64_t>(c->d) / 64, 64, kPairHalfRows);
+        if (rc) {
+            cudaFree(wt);
+            return rc;
+        }
+        c->W_tiled = wt;
+    } else {
+        rc = encode_bf16_2d(&m2, W_head, static_cast<uint64_t>(c->V), c->d, kPairHalfRows);
+        if (rc) return rc;
+    }
     c->maps.w128 = m2;
     c->W = W_head;
     c->g = g_norm;
@@ -581,6 +611,14 @@ int rpd_set_projection(rpd_ctx *c, int mode) {
     if (mode != RPD_PROJECT_ALL && mode != RPD_PROJECT_LAZY && mode != RPD_PROJECT_AUTO)
         return fail(RPD_ERR_INVALID_ARGUMENT, "unknown projection mode %d", mode);
     c->projection = mode;
+    return RPD_OK;
+}
+
+int rpd_set_head_layout(rpd_ctx *c, int layout) {
+    if (!c) return fail(RPD_ERR_INVALID_ARGUMENT, "null context");
+    if (layout != RPD_HEAD_TILED && layout != RPD_HEAD_BORROWED)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "unknown head layout %d", layout);
+    c->head_layout = layout;
     return RPD_OK;
 }
 
@@ -742,7 +780,7 @@ int rpd_step_shard_partials(rpd_ctx *c, const void *hidden, const uint8_t *mask,
     }
     if (e == cudaSuccess) {
         HeadParams hp{c->inv_rms, c->partials, c->meta, c->V, c->d, c->max_splits, c->wait_limit_ns,
-                      c->stall_next ? 1 : 0};
+                      c->stall_next ? 1 : 0, c->W_tiled != nullptr ? 1 : 0};
         e = launch_head(c->maps, hp, c->head_grid, c->stream);
         c->stall_next = false;
     }
@@ -826,6 +864,7 @@ void rpd_destroy(rpd_ctx *c) {
     DeviceGuard dg(c->device);
     cudaStreamSynchronize(c->stream);
     c->free_scratch();
+    if (c->W_tiled) cudaFree(c->W_tiled);
     if (c->stage) cudaFree(c->stage);
     if (c->stage_host) cudaFreeHost(c->stage_host);
     for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);

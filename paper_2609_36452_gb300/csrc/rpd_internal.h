@@ -13,12 +13,12 @@ namespace rpd {
 
 // Head-statistics tiles (tcgen05 cta_group::2: a cluster of two CTAs, one per SM, M = 256).
 // Pair tiles: 256 rows x 256 vocabulary columns per pair; each CTA stages its own 128 rows of
-// u and 128 rows of W per K-step of 64 (32 KB), 6 stages deep.
+// u and 128 rows of W per K-step of 64 (32 KB), 7 stages deep.
 constexpr int kTileM = 128;   // rows of u per CTA (TMEM lanes) and the row padding unit of scratch
 constexpr int kTileN = 256;   // vocabulary entries per tile
 constexpr int kTileK = 64;
 constexpr int kPairTileM = 256;
-constexpr int kPairStages = 6;
+constexpr int kPairStages = 7;
 constexpr int kPairHalfRows = 128;
 constexpr int kPairStageBytesA = kPairHalfRows * kTileK * 2;
 constexpr int kPairStageBytesB = kPairHalfRows * kTileK * 2;
@@ -32,21 +32,19 @@ constexpr int kSwapRowStep = 32;  // N of the M = 256 MMA: a multiple of 32, at 
 constexpr int kSwapMaxStages = 12;
 constexpr int kSwapStageBytesA = kPairHalfRows * kTileK * 2;
 
-constexpr int kSwapEpiWarps = 4;   // one per TMEM sub-partition, each taking all its chunks
+constexpr int kSwapEpiWarps = 8;   // two per TMEM sub-partition, alternating its chunks
 constexpr int kSwapXposeStride = 33;                             // floats per padded row
 constexpr int kSwapXposeBytes = kSwapEpiWarps * 32 * kSwapXposeStride * 4;  // 32 x 32 fp32 per warp
 // rows on N: running statistics [sub-partition][row of the group], 4 * ng float4
 constexpr int kUBoxRows = 16;  // granularity of a half group's rows (the TMA box heights)
-// Roles: warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-5 epilogue.  Six warps keep the kernel's
-// registers to about half of an SM's, so that the CTAs of the next kernel in the stream (launched
-// early, waiting on this grid) can already be resident when it finishes.
+// Roles: warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-9 epilogue (pair tiles use warps 2-5).
+// At 128 registers a thread the CTA holds 40 K of an SM's 64 K registers, which leaves room for
+// a CTA of the next kernel in the stream (launched early, waiting on this grid).
 constexpr int kHeadKernelThreads = 64 + 32 * kSwapEpiWarps;
 constexpr int kHeadBarrierBytes = 512;
 // The pair tiles' operand ring, or the rows-on-N ring, transpose blocks and statistics (the
-// ring takes what the other two leave).  The kernel keeps to about the pair ring's 192 KB: its
-// CTAs become resident (waiting) while the step's gather kernel still runs, and a larger
-// footprint leaves fewer gather CTAs room beside them (measured ~3 us a step at 211 KB).
-constexpr int kHeadRegionBytes = 193 * 1024;
+// ring takes what the other two leave): the 7-stage pair ring, 224 KB.
+constexpr int kHeadRegionBytes = 224 * 1024;
 static_assert(kPairStages * (kPairStageBytesA + kPairStageBytesB) <= kHeadRegionBytes,
               "the pair tiles' operand ring fits the region");
 static_assert(kHeadRegionBytes - kSwapXposeBytes - 4 * kSwapMaxRows * 16 >=
@@ -203,6 +201,7 @@ struct HeadParams {
     int V, d, max_splits;
     uint64_t wait_limit_ns;  // bound on every mbarrier wait
     int stall;               // diagnostics: issue no loads (the waits run out)
+    int w_tiled;             // W is the context's tiled copy (rpd_set_head_layout), else row-major
 };
 
 // Time to stream the head once, in units of one 128 x 256 tile's MMA time on one SM.
@@ -312,6 +311,9 @@ struct HeadMaps {
 // The head kernel (every tiling; the pass's choice is read from the meta words), launched as
 // `grid` CTAs in clusters of two, one per SM.
 cudaError_t launch_head(const HeadMaps &maps, const HeadParams &p, int grid, cudaStream_t s);
+// Copy W [V][d] (d % 64 == 0) into blocks of 128 rows x 64 columns, block (t, k) at element
+// ((t * (d / 64) + k) * 128) * 64, rows past V zero; Wt holds ceil(V/128)*128*d elements.
+cudaError_t launch_tile_head(const void *W, void *Wt, int V, int d, cudaStream_t s);
 // Largest number of clusters of the head kernel that can be resident at once.
 int head_max_clusters();
 cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t *sel_list,

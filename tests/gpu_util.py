@@ -13,7 +13,8 @@ def bits(t: torch.Tensor) -> np.ndarray:
 class DeviceRunner:
     """Context + head on cuda:0; runs single or batched steps with every debug output."""
 
-    def __init__(self, W: torch.Tensor, g: torch.Tensor, K: int, eps: float = 1e-6, rule="llada"):
+    def __init__(self, W: torch.Tensor, g: torch.Tensor, K: int, eps: float = 1e-6, rule="llada",
+                 layout=None):
         import paper_2609_36452_gb300 as rpd
         self.rpd = rpd
         self.dev = torch.device("cuda:0")
@@ -22,6 +23,8 @@ class DeviceRunner:
         self.W = W.to(self.dev).contiguous()
         self.g = g.to(self.dev).contiguous()
         self.ctx = rpd.Rpd(self.d, self.V, K, eps)
+        if layout is not None:
+            self.ctx.set_head_layout(layout)
         self.ctx.set_head(self.W, self.g)
         self.set_rule(rule)
         self.ctx.set_stream(torch.cuda.current_stream(self.dev))

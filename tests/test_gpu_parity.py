@@ -130,6 +130,31 @@ def test_head_tilings_match_oracle(tiling, d, V, K, N, frac):
 
 
 @pytest.mark.parametrize("tiling", ["pair", "rows_n"])
+@pytest.mark.parametrize("d,V,K,N", [
+    (256, 4100, 3, 100),    # ragged last vocabulary block (4100 = 32 x 128 + 4)
+    (4096, 1280, 2, 150),   # 64 column blocks per row block
+    (192, 2100, 4, 300),    # 1200 rows: several row tiles / two groups
+])
+def test_head_layouts_give_identical_outputs(tiling, d, V, K, N):
+    """The context's tiled copy of the head and the caller's row-major head feed the MMAs the
+    same operands in the same order, so every output is bitwise the same."""
+    case = small_case(1300 + d + K, K=K, N=N, d=d, V=V, w_std=0.08)
+    outs = {}
+    for layout in ("tiled", "borrowed"):
+        runner = DeviceRunner(case["W"], case["g"], K, case["eps"], rule=case["rule"], layout=layout)
+        try:
+            runner.ctx.set_head_tiling(tiling)
+            outs[layout] = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+        finally:
+            runner.close()
+    a, b = outs["tiled"], outs["borrowed"]
+    assert a["stats"] == b["stats"]
+    for k in a:
+        if k != "stats":
+            assert np.array_equal(a[k], b[k]), k
+
+
+@pytest.mark.parametrize("tiling", ["pair", "rows_n"])
 @pytest.mark.parametrize("rows", [1, 64, 127, 128, 129, 257, 320, 383, 384, 385, 513, 769, 832,
                                   895, 896, 897, 1023, 1025])
 def test_row_counts_around_tile_boundaries(tiling, rows):
