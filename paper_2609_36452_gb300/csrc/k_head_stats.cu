@@ -452,8 +452,9 @@ __device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, volatil
 // in shared memory).  At the end of a work unit the four sub-partitions' statistics of each
 // row are combined and each CTA writes one partial per row (the merge sees 2 partials per
 // split).
-// Each MMA's share of u in a stage is one TMA copy, from the tensor map whose box has that
-// share's height (16 to 128 rows).
+// Each CTA stages its half of the group (rows [r * G_r/2, +G_r/2)) as one TMA copy per stage,
+// from the tensor map whose box has that height (16 to 256 rows); the epilogue maps TMEM
+// columns back to rows (a stage with a second, small copy measured far slower).
 __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps] */,
                                           const CUtensorMap *tmW,
                                           const HeadParams &p, const HeadSmem &sm, int rows,
@@ -496,8 +497,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
         mbar_init(sm.drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&tmUrows[(n0 / 2) / kUBoxRows - 1]);
-        if (n1 > 0) tma_prefetch_desc(&tmUrows[(n1 / 2) / kUBoxRows - 1]);
+        tma_prefetch_desc(&tmUrows[(ng / 2) / kUBoxRows - 1]);
         tma_prefetch_desc(tmW);
     }
     if (warp == 1) tmem_alloc_pair(sm.tmem_slot, kTmemCols);
@@ -518,10 +518,10 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
             const uint32_t unit_full1 = mapa_shared(smem_u32(&unit_full[0]), 1);
             const uint32_t unit_ring1 = mapa_shared(smem_u32(const_cast<int *>(&unit_ring[0])), 1);
             const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
-            const int half0 = n0 / 2, half1 = n1 / 2;  // rows this CTA stages for each MMA
-            // one copy per MMA's share of u: the map whose box is that many rows high
-            const CUtensorMap *map0 = &tmUrows[half0 / kUBoxRows - 1];
-            const CUtensorMap *map1 = &tmUrows[(half1 > 0 ? half1 : kUBoxRows) / kUBoxRows - 1];
+            // this CTA's half of the group's rows, one copy: the map whose box is that many rows
+            // high (rows [rank * half, +half) of the group; see the epilogue's row order)
+            const int half = ng / 2;
+            const CUtensorMap *umap = &tmUrows[half / kUBoxRows - 1];
             int stage = 0;
             uint32_t phase = 0;
             long long fills = 0;
@@ -550,8 +550,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                 if (u < 0) break;
                 int m, g, v0, v1;
                 tw.unit(u, m, g, v0, v1);
-                const int rows0 = m * ng + static_cast<int>(rank) * half0;
-                const int rows1 = m * ng + kPairTileM + static_cast<int>(rank) * half1;
+                const int urow = m * ng + static_cast<int>(rank) * half;
                 const int w_off = static_cast<int>(rank) * kPairHalfRows;
                 for (int n = v0; ok && n < v1; ++n) {
                     for (int kb = 0; kb < num_kb; ++kb) {
@@ -568,9 +567,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                                              ((2 * n + static_cast<int>(rank)) * num_kb + kb) * kPairHalfRows);
                         else
                             tma_load_2d_pair(st, tmW, fb, x, n * kTileN + w_off);
-                        uint8_t *sb = st + kSwapStageBytesA;
-                        tma_load_2d_pair(sb, map0, fb, x, rows0);
-                        if (half1 > 0) tma_load_2d_pair(sb + half0 * (kTileK * 2), map1, fb, x, rows1);
+                        tma_load_2d_pair(st + kSwapStageBytesA, umap, fb, x, urow);
                         ++fills;
                         if (++stage == stages) {
                             stage = 0;
@@ -699,8 +696,15 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = xp[i * kSwapXposeStride + lane];
                     __syncwarp();
-                    // now v[i] = logit of vocabulary entry vbase + i for row c*32 + lane
-                    const int rl = c * 32 + lane;
+                    // now v[i] = logit of vocabulary entry vbase + i for TMEM column c*32 + lane,
+                    // i.e. for row rl of the group: MMA j takes its first N_j/2 columns from the
+                    // even CTA's rows [o_j, o_j + N_j/2) and the rest from the odd CTA's, and CTA r
+                    // holds the group's rows [r * ng/2, +ng/2) (o_0 = 0, o_1 = n0/2)
+                    const int col = c * 32 + lane;
+                    const int seg1 = col >= n0 ? 1 : 0;
+                    const int x = col - seg1 * n0;
+                    const int hj = seg1 ? n1 / 2 : n0 / 2;
+                    const int rl = seg1 * (n0 / 2) + (x < hj ? x : ng / 2 + (x - hj));
                     const int r = m * ng + rl;
                     const float scale = r < rows ? __ldg(p.inv_rms + r) * kLog2e : 0.f;
                     float4 st = stats[sub * ng + rl];

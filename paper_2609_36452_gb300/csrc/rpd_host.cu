@@ -213,9 +213,10 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
     if (bn <= c->cap_bn && B <= c->cap_b) return RPD_OK;
     const int new_bn = static_cast<int>(std::max<long long>(bn, c->cap_bn));
     const int new_b = std::max(B, c->cap_b);
+    // padded to whole pair tiles, so that every u box (at most 256 rows) fits in the tensor
     long long rows = static_cast<long long>(c->K) * new_bn;
-    rows = ((rows + kTileM - 1) / kTileM) * kTileM;
-    if (rows < kTileM) rows = kTileM;
+    rows = ((rows + kPairTileM - 1) / kPairTileM) * kPairTileM;
+    if (rows < kPairTileM) rows = kPairTileM;
     if (rows > (1ll << 30)) return fail(RPD_ERR_UNSUPPORTED, "too many projected rows (%lld)", rows);
     cudaError_t e = cudaStreamSynchronize(c->stream);  // no step may still use old scratch
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");

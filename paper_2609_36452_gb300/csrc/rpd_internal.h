@@ -302,7 +302,7 @@ cudaError_t launch_gather_norm(const NormParams &p, int grid, cudaStream_t s);
 // per half-group height, so that a stage copies each MMA's share of u with one instruction:
 // the TMA unit's time per copy, not its bytes, bounded a stage built from 16-row boxes); W in
 // boxes of 128 rows.
-constexpr int kUMaps = kPairHalfRows / kUBoxRows;  // box heights kUBoxRows * (1 .. kUMaps)
+constexpr int kUMaps = (kSwapMaxRows / 2) / kUBoxRows;  // box heights kUBoxRows * (1 .. kUMaps)
 struct HeadMaps {
     CUtensorMap u;                // box 64 x 128 rows
     CUtensorMap w128;             // box 64 x 128 rows of W
