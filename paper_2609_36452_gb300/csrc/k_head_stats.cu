@@ -148,6 +148,7 @@ struct HeadSmem {
     uint64_t *unit_full;      // [kUnitRing] producer -> MMA, epilogue
     uint64_t *unit_empty;     // [kUnitRing] MMA, epilogue -> producer
     uint64_t *epi;            // [1] rows-on-N tiling: barrier of the epilogue warps
+    uint64_t *chunk_free;     // [16] rows-on-N tiling: TMEM chunk read (in the even CTA)
     uint32_t *tmem_slot;
     volatile int *abort_flag;
     volatile int *unit_ring;  // [kUnitRing] claimed unit indices
@@ -167,13 +168,15 @@ __device__ __forceinline__ HeadSmem carve_smem(uint8_t *raw) {
     s.unit_full = s.drain + 1;
     s.unit_empty = s.unit_full + kUnitRing;
     s.epi = s.unit_empty + kUnitRing;
-    s.tmem_slot = reinterpret_cast<uint32_t *>(s.epi + 1);
+    s.chunk_free = s.epi + 1;
+    s.tmem_slot = reinterpret_cast<uint32_t *>(s.chunk_free + kTmemCols / 32);
     s.abort_flag = reinterpret_cast<volatile int *>(s.tmem_slot + 1);
     s.unit_ring = s.abort_flag + 1;
     return s;
 }
 
-static_assert((2 * kSwapMaxStages + 6 + 2 * kUnitRing) * 8 + 8 + 4 * kUnitRing <= kHeadBarrierBytes,
+static_assert((2 * kSwapMaxStages + 6 + 2 * kUnitRing + kTmemCols / 32) * 8 + 8 + 4 * kUnitRing <=
+                  kHeadBarrierBytes,
               "barrier region");
 
 // ------------------------------------------------------------------------------------------
@@ -440,36 +443,104 @@ __device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, volatil
 // ------------------------------------------------------------------------------------------
 // Tiling 2: "rows on N" CTA pairs.  The pair's MMA (cta_group::2, M = 256) takes the head as
 // its A operand - CTA r stages vocabulary rows [256n + 128r, +128) of tile n, 16 KB per
-// K-step - and a group of G_r rows of u as its B operand (N = G_r, a multiple of 32 up to
-// 512): the first N/2 columns come from the even CTA's shared memory, the rest from the odd
-// CTA's.  A group of more than 256 rows is issued as two MMAs (N = 256 and N = G_r - 256,
-// TMEM columns [0, 256) and [256, G_r)); a group of at most 256 rows is double-buffered in
-// TMEM.  So CTA r's TMEM holds logits for 128 vocabulary entries (lanes) x the group's rows
-// (columns): per row the softmax statistics reduce across lanes.  The epilogue (4 warps, one
-// per TMEM sub-partition, each taking every 32-column chunk of its lanes) loads a 32 x 32
-// block, transposes it through shared memory so that each thread holds one row's 32
-// vocabulary entries, and folds them into that row's running statistics (per sub-partition,
-// in shared memory).  At the end of a work unit the four sub-partitions' statistics of each
-// row are combined and each CTA writes one partial per row (the merge sees 2 partials per
-// split).
-// Each CTA stages its half of the group (rows [r * G_r/2, +G_r/2)) as one TMA copy per stage,
-// from the tensor map whose box has that height (16 to 256 rows); the epilogue maps TMEM
-// columns back to rows (a stage with a second, small copy measured far slower).
+// K-step - and a group of G rows of u as its B operand (N = G, a multiple of 32 up to 512).
+// So CTA r's TMEM holds logits for 128 vocabulary entries (lanes) x the group's rows
+// (columns): per row the softmax statistics reduce across lanes.
+//
+// Operands: each CTA stages its half of the group (rows [r G/2, +G/2)) as one TMA copy per
+// stage, from the tensor map whose box has that height (16 to 256 rows; a stage with a second,
+// small copy measured far slower).
+//
+// TMEM: 16 chunks of 32 columns.  A tile of at most 256 columns alternates between the two
+// halves (double buffering); a tile of 288 or 320 columns follows its predecessor around the
+// ring of chunks, so that it waits only for the chunks it overwrites (with 288 columns, the
+// first two of its predecessor's nine) instead of for the whole epilogue of its predecessor;
+// larger tiles use columns [0, G) in turn.  A tile's columns are issued as one MMA per
+// contiguous segment of at most 256 columns per 16-wide K-step, and the MMA for columns
+// [c, c + N) of segment j takes the first N/2 of them from rows [o_j, o_j + N/2) of the even
+// CTA's half and the rest from the same rows of the odd CTA's half, o_j being half the columns
+// of the tile before segment j; the epilogue maps each column back to its row.
+//
+// Epilogue: 8 warps, two per TMEM sub-partition, alternating its chunks.  A warp loads a
+// 32 x 32 block, releases the chunk (ring tiles), transposes the block through shared memory
+// so that each thread holds one row's 32 vocabulary entries, and folds them into that row's
+// running statistics (per sub-partition, in shared memory).  At the end of a work unit the
+// four sub-partitions' statistics of each row are combined and each CTA writes one partial
+// per row (the merge sees 2 partials per split).
+// The K-steps of one rows-on-N tile issued as kSegs MMAs per 16-wide step (one per column
+// segment).  A separate loop per segment count keeps the issuing thread's loop free of
+// branches: with the segment tests inside the loop the single issuing thread measured 60 %
+// slower per tile.
+template <int kSegs>
+__device__ __forceinline__ bool swap_tile_mmas(const HeadSmem &sm, int num_kb, int stages,
+                                               int stage_bytes, int &stage, uint32_t &phase,
+                                               uint32_t d0, uint32_t d1, uint32_t d2, uint32_t id0,
+                                               uint32_t id1, uint32_t id2, uint32_t bo1,
+                                               uint32_t bo2, volatile int *abort_flag,
+                                               uint64_t limit) {
+    for (int kb = 0; kb < num_kb; ++kb) {
+        if (!mbar_wait_bounded(&sm.full[stage], phase, abort_flag, limit)) return false;
+        tc_fence_after_sync();
+        const uint32_t a0 = smem_u32(sm.ring + stage * stage_bytes);
+        const uint32_t b0 = a0 + kSwapStageBytesA;
+#pragma unroll
+        for (int kk = 0; kk < kTileK / 16; ++kk) {
+            const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
+            umma_bf16_pair(d0, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + kk * 32), id0, accum);
+            if (kSegs > 1)
+                umma_bf16_pair(d1, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + bo1 + kk * 32),
+                               id1, accum);
+            if (kSegs > 2)
+                umma_bf16_pair(d2, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + bo2 + kk * 32),
+                               id2, accum);
+        }
+        umma_commit_pair_multicast(&sm.empty[stage], 0x3);
+        if (++stage == stages) {
+            stage = 0;
+            phase ^= 1u;
+        }
+    }
+    return true;
+}
+
+// Column segments of a rows-on-N tile placed at TMEM chunk c0: up to three contiguous column
+// ranges, each within [0, 512) and at most 256 wide (the MMA's N).
+struct SwapSegs {
+    int col0, col1, col2;  // first TMEM column of each
+    int n0, n1, n2;        // widths (0: unused)
+};
+__device__ __forceinline__ SwapSegs swap_segments(int c0, int ng) {
+    SwapSegs g;
+    g.col0 = c0 * 32;
+    g.n0 = min(min(ng, kTmemCols - g.col0), kPairTileM);
+    g.col1 = (g.col0 + g.n0) % kTmemCols;
+    g.n1 = min(min(ng - g.n0, kTmemCols - g.col1), kPairTileM);
+    g.col2 = (g.col1 + g.n1) % kTmemCols;
+    g.n2 = ng - g.n0 - g.n1;
+    return g;
+}
+
 __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps] */,
                                           const CUtensorMap *tmW,
                                           const HeadParams &p, const HeadSmem &sm, int rows,
                                           int splits, int ng) {
     uint64_t *full = sm.full, *empty = sm.empty, *acc_full = sm.acc_full,
-             *acc_empty = sm.acc_empty, *unit_full = sm.unit_full, *unit_empty = sm.unit_empty;
+             *acc_empty = sm.acc_empty, *unit_full = sm.unit_full, *unit_empty = sm.unit_empty,
+             *chunk_free = sm.chunk_free;
     volatile int *abort_flag = sm.abort_flag;
     volatile int *unit_ring = sm.unit_ring;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const uint32_t rank = cluster_ctarank();
-    // group geometry: columns of the two MMAs, accumulator buffers, ring depth
-    const int n0 = ng < kPairTileM ? ng : kPairTileM;
-    const int n1 = ng - n0;
-    const int nbuf = ng <= kPairTileM ? 2 : 1;
+    // TMEM placement: tiles of at most 256 columns alternate between the two halves; tiles of
+    // 288 to 320 columns follow one another around a ring of 16 chunks of 32 columns; larger
+    // tiles use all of TMEM in turn (with 11 or more chunks a tile would wait for nearly all of
+    // its predecessor's chunks anyway, and the ring's column splits measured slower there)
+    constexpr uint32_t kChunks = kTmemCols / 32;
+    constexpr uint32_t kRingMaxChunks = 10;
+    const uint32_t nch = static_cast<uint32_t>(ng / 32);
+    const bool single = nch > kRingMaxChunks;
+    const bool ring = 2 * nch > kChunks && !single;
     const int stage_b = (ng / 2) * kTileK * 2;
     const int stage_bytes = kSwapStageBytesA + stage_b;
     // region: operand ring (as many stages as fit), transpose blocks, statistics [4][ng]
@@ -493,6 +564,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
             // even CTA: its MMA issuer and epilogue warps; odd CTA: its producer and epilogue warps
             mbar_init(&unit_empty[i], 2 + 2 * kSwapEpiWarps);
         }
+        for (uint32_t i = 0; i < kChunks; ++i) mbar_init(&chunk_free[i], 8);
         mbar_init(sm.epi, kEpiThreads);
         mbar_init(sm.drain, 1);
         *abort_flag = 0;
@@ -586,9 +658,6 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
         if (lane == 0) {
             if (rank == 0) {
                 // ------------------------------------------------ MMA issuer (even CTA only)
-                const uint32_t idesc0 = idesc_bf16_f32(kPairTileM, n0);
-                const uint32_t idesc1 = idesc_bf16_f32(kPairTileM, n1 > 0 ? n1 : 16);
-                const uint32_t b1_off = static_cast<uint32_t>((n0 / 2) * kTileK * 2);
                 int stage = 0;
                 uint32_t phase = 0;
                 uint32_t tile_iter = 0;
@@ -604,38 +673,46 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                     int m, g, v0, v1;
                     tw.unit(u, m, g, v0, v1);
                     for (int n = v0; ok && n < v1; ++n, ++tile_iter) {
-                        const uint32_t acc = nbuf == 2 ? (tile_iter & 1u) : 0u;
-                        const uint32_t acc_phase = (nbuf == 2 ? (tile_iter >> 1) : tile_iter) & 1u;
+                        // tile t-2 read (its accumulator barrier is reused), or tile t-1 for tiles
+                        // that use all of TMEM ...
+                        const uint32_t acc = single ? 0u : (tile_iter & 1u);
+                        const uint32_t acc_phase = (single ? tile_iter : (tile_iter >> 1)) & 1u;
                         if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
                                                p.wait_limit_ns)) {
                             ok = false;
                             break;
                         }
-                        tc_fence_after_sync();
-                        const uint32_t d_tmem = tmem_base + acc * kTileN;
-                        for (int kb = 0; kb < num_kb; ++kb) {
-                            if (!mbar_wait_bounded(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
-                                ok = false;
-                                break;
+                        // ... and, on the ring, the chunks of tile t-1 this tile overwrites
+                        const uint32_t a0 = tile_iter * nch;
+                        if (ring && tile_iter > 0) {
+                            for (uint32_t c = kChunks - nch; ok && c < nch; ++c) {
+                                const uint32_t a = a0 + c;  // previous use: a - 16, in tile t-1
+                                if (!mbar_wait_bounded(&chunk_free[a % kChunks], ((a / kChunks) & 1u) ^ 1u,
+                                                       abort_flag, p.wait_limit_ns))
+                                    ok = false;
                             }
-                            tc_fence_after_sync();
-                            const uint32_t a0 = smem_u32(sm.ring + stage * stage_bytes);
-                            const uint32_t b0 = a0 + kSwapStageBytesA;
-#pragma unroll
-                            for (int kk = 0; kk < kTileK / 16; ++kk) {
-                                const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
-                                umma_bf16_pair(d_tmem, smem_desc_sw128(a0 + kk * 32),
-                                               smem_desc_sw128(b0 + kk * 32), idesc0, accum);
-                                if (n1 > 0)
-                                    umma_bf16_pair(d_tmem + kPairTileM, smem_desc_sw128(a0 + kk * 32),
-                                                   smem_desc_sw128(b0 + b1_off + kk * 32), idesc1, accum);
-                            }
-                            umma_commit_pair_multicast(&empty[stage], 0x3);
-                            if (++stage == stages) {
-                                stage = 0;
-                                phase ^= 1u;
-                            }
+                            if (!ok) break;
                         }
+                        tc_fence_after_sync();
+                        const SwapSegs sg = swap_segments(static_cast<int>(ring ? a0 % kChunks : acc * 8u), ng);
+                        // (single: acc = 0, the tile starts at column 0)
+                        const uint32_t d0 = tmem_base + sg.col0, d1 = tmem_base + sg.col1,
+                                       d2 = tmem_base + sg.col2;
+                        const uint32_t id0 = idesc_bf16_f32(kPairTileM, sg.n0);
+                        const uint32_t id1 = idesc_bf16_f32(kPairTileM, sg.n1 > 0 ? sg.n1 : 32);
+                        const uint32_t id2 = idesc_bf16_f32(kPairTileM, sg.n2 > 0 ? sg.n2 : 32);
+                        // segment j's rows of u start at row (columns before it) / 2 of each CTA's half
+                        const uint32_t bo1 = static_cast<uint32_t>((sg.n0 / 2) * kTileK * 2);
+                        const uint32_t bo2 = static_cast<uint32_t>(((sg.n0 + sg.n1) / 2) * kTileK * 2);
+                        ok = sg.n2 > 0 ? swap_tile_mmas<3>(sm, num_kb, stages, stage_bytes, stage, phase, d0, d1,
+                                                           d2, id0, id1, id2, bo1, bo2, abort_flag,
+                                                           p.wait_limit_ns)
+                           : sg.n1 > 0 ? swap_tile_mmas<2>(sm, num_kb, stages, stage_bytes, stage, phase, d0,
+                                                           d1, d2, id0, id1, id2, bo1, bo2, abort_flag,
+                                                           p.wait_limit_ns)
+                                       : swap_tile_mmas<1>(sm, num_kb, stages, stage_bytes, stage, phase, d0,
+                                                           d1, d2, id0, id1, id2, bo1, bo2, abort_flag,
+                                                           p.wait_limit_ns);
                         if (!ok) break;
                         umma_commit_pair_multicast(&acc_full[acc], 0x3);
                     }
@@ -650,9 +727,9 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
         const int etid = (warp - 2) * 32 + lane;  // 0 .. kEpiThreads-1
         const int chunk0 = (warp - 2) / 4;        // the two warps of a sub-partition alternate chunks
         constexpr int kChunkStep = kSwapEpiWarps / 4;
-        const int nch = ng / 32;
         const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
         const uint32_t acc_empty0 = mapa_shared(smem_u32(&acc_empty[0]), 0);
+        const uint32_t chunk_free0 = mapa_shared(smem_u32(&chunk_free[0]), 0);
         const uint32_t unit_empty0 = mapa_shared(smem_u32(&unit_empty[0]), 0);
         float *xp = xpose + (warp - 2) * 32 * kSwapXposeStride;
         const float4 kEmpty = make_float4(-INFINITY, 0.f, 0.f, __int_as_float(0));
@@ -673,20 +750,29 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
             int m, g, v0, v1;
             tw.unit(u, m, g, v0, v1);
             for (int n = v0; n < v1; ++n, ++tile_iter) {
-                const uint32_t acc = nbuf == 2 ? (tile_iter & 1u) : 0u;
-                const uint32_t acc_phase = (nbuf == 2 ? (tile_iter >> 1) : tile_iter) & 1u;
+                const uint32_t acc = single ? 0u : (tile_iter & 1u);
+                const uint32_t acc_phase = (single ? tile_iter : (tile_iter >> 1)) & 1u;
                 if (!mbar_wait_bounded(&acc_full[acc], acc_phase, abort_flag, p.wait_limit_ns)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after_sync();
+                const uint32_t c0 = ring ? (tile_iter * nch) % kChunks : acc * 8u;
+                const SwapSegs sg = swap_segments(static_cast<int>(c0), ng);
+                const int x1 = sg.n0, x2 = sg.n0 + sg.n1;
                 // the 32 vocabulary entries of this warp's sub-partition
                 const int vbase = n * kTileN + static_cast<int>(rank) * kPairHalfRows + sub * 32;
                 const bool full_tile = vbase + 32 <= p.V;
 #pragma unroll 1
-                for (int c = chunk0; c < nch; c += kChunkStep) {
+                for (int c = chunk0; c < static_cast<int>(nch); c += kChunkStep) {
                     float v[32];
-                    tmem_ld_32x32b_x32(lane_base + acc * kTileN + c * 32, v);
+                    const uint32_t slot = (c0 + static_cast<uint32_t>(c)) % kChunks;
+                    tmem_ld_32x32b_x32(lane_base + slot * 32, v);
+                    if (ring) {  // the chunk's columns may be overwritten by the next tile now
+                        tc_fence_before_sync();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive_cluster(chunk_free0 + slot * static_cast<uint32_t>(sizeof(uint64_t)));
+                    }
                     // thread `lane` holds vocabulary entry vbase + lane for rows c*32 + i; write
                     // it as row `lane` of a block padded to 33 floats a row (bank lane + i: no
                     // conflict) and read back column `lane` (bank i + lane: no conflict)
@@ -700,11 +786,11 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                     // i.e. for row rl of the group: MMA j takes its first N_j/2 columns from the
                     // even CTA's rows [o_j, o_j + N_j/2) and the rest from the odd CTA's, and CTA r
                     // holds the group's rows [r * ng/2, +ng/2) (o_0 = 0, o_1 = n0/2)
-                    const int col = c * 32 + lane;
-                    const int seg1 = col >= n0 ? 1 : 0;
-                    const int x = col - seg1 * n0;
-                    const int hj = seg1 ? n1 / 2 : n0 / 2;
-                    const int rl = seg1 * (n0 / 2) + (x < hj ? x : ng / 2 + (x - hj));
+                    const int col = c * 32 + lane;  // column of the tile
+                    const int xj = col < x1 ? 0 : (col < x2 ? x1 : x2);
+                    const int nj = col < x1 ? sg.n0 : (col < x2 ? sg.n1 : sg.n2);
+                    const int x = col - xj;
+                    const int rl = xj / 2 + (x < nj / 2 ? x : ng / 2 + (x - nj / 2));
                     const int r = m * ng + rl;
                     const float scale = r < rows ? __ldg(p.inv_rms + r) * kLog2e : 0.f;
                     float4 st = stats[sub * ng + rl];
