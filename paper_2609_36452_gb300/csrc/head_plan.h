@@ -57,7 +57,8 @@ __host__ __device__ inline unsigned long long best_split_key(float tile_cost, in
 // Time of one "rows on N" tile (256 vocabulary entries x a group of `ng` rows on a CTA pair)
 // in tile units (the measured calibration of rpd_internal.h).
 __host__ __device__ inline float swap_tile_cost(int ng) {
-    return kSwapTileBase + kSwapTilePerRow * static_cast<float>(ng);
+    return ng <= kPairTileM ? kSwapTileBase + kSwapTilePerRow * static_cast<float>(ng)
+                            : kSwapWideTileBase + kSwapWideTilePerRow * static_cast<float>(ng);
 }
 
 // Rows-on-N groups of a pass: as few as possible (every group streams the whole head through
@@ -72,24 +73,24 @@ __host__ __device__ inline int swap_group_rows(long long rows, int groups) {
 }
 
 // The plan from the best keys of both tilings: each estimate is the larger of its MMA time and
-// the head streaming time scaled by the vocabulary share of its largest split; the cheaper wins
-// (equal estimates - both bound by streaming the head - go to the one with less MMA work), or
-// the one `force` names.
+// the head streaming time scaled by the vocabulary share of its largest split (and, for pair
+// tiles, by their slower streaming); the cheaper wins (equal estimates go to the one with less
+// MMA work), or the one `force` names.
 __host__ __device__ inline HeadPlan plan_from_keys(const HeadPlanInputs &in, unsigned long long key2,
                                                    unsigned long long key3, int ng3) {
-    auto est_of = [&](float t, int g) {
+    auto est_of = [&](float t, int g, float stream) {
         const float per = static_cast<float>((in.num_n + g - 1) / g);
-        const float hbm = in.hbm_tiles * per * static_cast<float>(g) / static_cast<float>(in.num_n);
+        const float hbm = stream * in.hbm_tiles * per * static_cast<float>(g) / static_cast<float>(in.num_n);
         return t > hbm ? t : hbm;
     };
     const int g2 = static_cast<int>(key2 & 0xFFFFFull);
     const float t2 = bits_float(static_cast<unsigned>(key2 >> 20));
-    const float e2 = est_of(t2, g2);
+    const float e2 = est_of(t2, g2, kPairStreamFactor);
     HeadPlan pair{kHeadModePair, g2, 0, e2};
     if (key3 == ~0ull || in.force == RPD_TILING_PAIR) return pair;
     const int g3 = static_cast<int>(key3 & 0xFFFFFull);
     const float t3 = bits_float(static_cast<unsigned>(key3 >> 20));
-    const float e3 = est_of(t3, g3);
+    const float e3 = est_of(t3, g3, 1.f);
     const bool rows_n = in.force == RPD_TILING_ROWS_N || e3 < e2 || (e3 == e2 && t3 < t2);
     return rows_n ? HeadPlan{kHeadModeRowsN, 2 * g3, ng3, e3} : pair;
 }

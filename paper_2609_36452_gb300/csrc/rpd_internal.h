@@ -165,15 +165,20 @@ struct BandParams {
 };
 
 // Costs of the tiling choice are in units of one 128-row x 256-entry tile's MMA work on one SM
-// at the nominal rate below.  Both tilings are bound less by the MMAs than by how many operand
-// bytes an SM can keep in flight against the latency of its copies (a ring of ~192 KB against
-// ~2.5 us on GB300), so the per-tile costs are measured ones (LLaDA head, d = 4096, GB300):
-//   pair tile (256 rows x 256 entries per pair): 23.6 us, 0.97 units;
-//   rows-on-N tile (256 entries x a group of ng rows): about 0.80 + 0.0027 ng units, i.e.
-//   19.5 + 0.066 ng us (96 rows: 25 us, 288: 38 us, 384: 46 us, 448: 46 us, 512: 51 us).
-constexpr float kPairTileCost = 0.97f;
-constexpr float kSwapTileBase = 0.80f;
-constexpr float kSwapTilePerRow = 0.0027f;
+// at the nominal rate below (24.4 us).  The per-tile costs are measured ones (LLaDA head,
+// d = 4096, GB300, head time / tiles per pair, both tilings forced at 20 to 1024 rows):
+//   pair tile (256 rows x 256 entries per pair): 23.0 us, 0.943 units;
+//   rows-on-N tile (256 entries x a group of ng rows): 21.6 + 0.023 ng us (0.885 + 0.00094 ng
+//   units) for ng <= 256, whose accumulators are double-buffered, and 12.6 + 0.074 ng us
+//   (0.516 + 0.00303 ng units) for larger groups (288 rows: 34 us, 416: 43 us, 512: 50 us).
+// When streaming the head bounds a pass, pair tiles - half of whose staged bytes are rows of u -
+// stream it about 5 % slower than rows-on-N tiles (20 rows: 0.163 against 0.155 ms).
+constexpr float kPairTileCost = 0.943f;
+constexpr float kSwapTileBase = 0.885f;
+constexpr float kSwapTilePerRow = 0.00094f;
+constexpr float kSwapWideTileBase = 0.516f;
+constexpr float kSwapWideTilePerRow = 0.00303f;
+constexpr float kPairStreamFactor = 1.05f;
 // Per-SM MMA rate of the unit tile and the sustained HBM read rate used by the tiling choice
 // (GB300 measurements; only their ratio matters).
 constexpr double kSingleTileFlopsPerSm = 1.1e13;
