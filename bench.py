@@ -518,6 +518,10 @@ def emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e, st
                 "frac": achieved / peak, "traffic": None, "peak_kind": f"HBM copy, of {peaks['source']}",
                 "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS}
     step_roof = max(t_tc, t_hbm) / (ms_step * 1e-3)
+    if roof["frac"] > 1.0:
+        # the denominators are measured rates (a cuBLAS GEMM, a copy kernel), not hardware
+        # limits: a kernel can exceed them a little, far more would mean skipped work
+        roof["above_measured_peak"] = True
     roof["traffic"] = HEAD_TRAFFIC.get((case["name"], head_source_hash()))
     roof["algorithmic_bytes"] = bytes_
     roof["algorithmic_flops"] = flops

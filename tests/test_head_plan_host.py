@@ -1,0 +1,103 @@
+"""The head-tiling plan on the host (no GPU): `csrc/head_plan.h` compiled with the host C++
+compiler and evaluated for every row count of a pass up to 4096 at the LLaDA-8B head shape on
+152 SMs.  Checks the plan's invariants, that a forced tiling is honoured, and that the automatic
+choice is the tiling measured faster on GB300 at the calibration row counts (both tilings
+forced, head kernel time per pass)."""
+import os
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+CSRC = os.path.join(ROOT, "paper_2609_36452_gb300", "csrc")
+
+# V, d of the LLaDA-8B head; 152 SMs -> 76 CTA pairs, at most 2 * SMs vocabulary splits
+V, D, SMS = 126464, 4096, 152
+NUM_N = (V + 255) // 256
+MAX_SPLITS = min(2 * NUM_N, 2 * SMS)
+PAIR, ROWS_N = 2, 3
+MAX_ROWS = 4096
+
+DRIVER = r"""
+#include "head_plan.h"
+#include <cstdio>
+int main() {
+    for (int force = 0; force <= 2; ++force) {
+        rpd::HeadPlanInputs in{};
+        in.num_n = %d; in.max_splits = %d; in.pair_slots = %d;
+        in.hbm_tiles = rpd::head_stream_in_tiles(%d, %d, %d);
+        in.force = force;
+        for (int r = 1; r <= %d; ++r) {
+            const rpd::HeadPlan p = rpd::plan_head(r, in);
+            std::printf("%%d %%d %%d %%d %%d %%.6f\n", force, r, p.mode, p.splits, p.swap_rows, p.est);
+        }
+    }
+    return 0;
+}
+""" % (NUM_N, MAX_SPLITS, SMS // 2, V, D, SMS, MAX_ROWS)
+
+# Measured on GB300 (LLaDA head, 200 steps per point): head kernel ms with pair tiles forced,
+# with rows-on-N tiles forced.  Where the two are within 1 %, either choice is accepted.
+MEASURED = {20: (0.1628, 0.1548), 64: (0.1648, 0.1581), 108: (0.1664, 0.1655),
+            160: (0.1692, 0.1713), 224: (0.1748, 0.1873), 256: (0.1776, 0.1932),
+            280: (0.2779, 0.2372), 320: (0.2801, 0.2514), 360: (0.2832, 0.2754),
+            428: (0.2914, 0.3273), 512: (0.2997, 0.3529), 600: (0.4275, 0.4473),
+            788: (0.5794, 0.5618), 1024: (0.5973, 0.6554)}
+
+
+@pytest.fixture(scope="module")
+def plans(tmp_path_factory):
+    cxx = shutil.which("g++") or shutil.which("c++")
+    inc = "/usr/local/cuda/include"
+    if not cxx or not os.path.exists(os.path.join(inc, "cuda_runtime.h")):
+        pytest.skip("needs a host C++ compiler and the CUDA headers")
+    d = tmp_path_factory.mktemp("plan")
+    src, exe = d / "plan.cpp", d / "plan"
+    src.write_text(DRIVER)
+    r = subprocess.run([cxx, "-std=c++17", "-O1", "-I", inc, "-I", CSRC, "-I",
+                        os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    table = {}
+    for line in out.split("\n"):
+        if line:
+            f, rows, mode, splits, swap_rows, est = line.split()
+            table[(int(f), int(rows))] = (int(mode), int(splits), int(swap_rows), float(est))
+    return table
+
+
+def test_plan_invariants(plans):
+    for (force, rows), (mode, splits, swap_rows, est) in plans.items():
+        assert mode in (PAIR, ROWS_N)
+        assert 1 <= splits <= MAX_SPLITS and est > 0
+        if mode == PAIR:
+            assert splits <= NUM_N and swap_rows == 0
+        else:
+            # two partials per split (one per CTA); groups padded to a multiple of 32 rows,
+            # at most 512, as few groups as possible, each holding its share of the rows
+            assert splits % 2 == 0 and splits // 2 <= NUM_N
+            assert swap_rows % 32 == 0 and 32 <= swap_rows <= 512
+            groups = -(-rows // 512)
+            assert swap_rows * groups >= rows and swap_rows - 32 < -(-rows // groups)
+
+
+def test_forced_tilings_are_honoured(plans):
+    for rows in range(1, MAX_ROWS + 1):
+        assert plans[(1, rows)][0] == PAIR
+        assert plans[(2, rows)][0] == ROWS_N
+
+
+def test_auto_picks_the_measured_faster_tiling(plans):
+    for rows, (t_pair, t_rows_n) in MEASURED.items():
+        mode = plans[(0, rows)][0]
+        if abs(t_pair - t_rows_n) <= 0.01 * min(t_pair, t_rows_n):
+            continue
+        assert mode == (PAIR if t_pair < t_rows_n else ROWS_N), rows
+
+
+def test_auto_is_the_cheaper_of_the_forced_estimates(plans):
+    for rows in range(1, MAX_ROWS + 1):
+        e_auto, e_pair, e_rows_n = plans[(0, rows)][3], plans[(1, rows)][3], plans[(2, rows)][3]
+        assert e_auto == pytest.approx(min(e_pair, e_rows_n), rel=1e-6)
