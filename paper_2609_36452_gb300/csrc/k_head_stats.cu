@@ -564,6 +564,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
             // even CTA: its MMA issuer and epilogue warps; odd CTA: its producer and epilogue warps
             mbar_init(&unit_empty[i], 2 + 2 * kSwapEpiWarps);
         }
+        // ring tiles: a chunk is read by one warp per TMEM sub-partition in each CTA
         for (uint32_t i = 0; i < kChunks; ++i) mbar_init(&chunk_free[i], 8);
         mbar_init(sm.epi, kEpiThreads);
         mbar_init(sm.drain, 1);
