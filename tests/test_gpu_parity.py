@@ -172,6 +172,23 @@ def test_row_counts_around_tile_boundaries(tiling, rows):
     print(compare_step(oracle_step(case), got))
 
 
+@pytest.mark.parametrize("rows", [280, 300, 320, 416])
+def test_rows_n_tmem_ring_with_several_tiles_per_pair(rows):
+    """Rows-on-N groups of 288 and 320 columns go round the ring of TMEM chunks (the second
+    tile of a CTA pair wraps at column 512 and waits for chunks of the first), 416 columns use
+    all of TMEM in turn.  A vocabulary of 60000 entries (235 tiles) gives every pair about three
+    tiles; every output is compared with the oracle."""
+    case = small_case(1500 + rows, K=1, N=rows, d=256, V=60000, w_std=0.08)
+    runner = DeviceRunner(case["W"], case["g"], 1, case["eps"], rule=case["rule"])
+    try:
+        runner.ctx.set_head_tiling("rows_n")
+        got = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+    finally:
+        runner.close()
+    assert got["stats"]["n_rows"] == rows
+    print(compare_step(oracle_step(case), got))
+
+
 @pytest.mark.parametrize("K,N", [(4, 70), (4, 107), (4, 128), (2, 300)])
 def test_rows_n_groups_with_window_layers(K, N):
     """The rows-on-N tiling with several window layers (rows are layer-major, so a group mixes
