@@ -154,6 +154,35 @@ def test_head_layouts_give_identical_outputs(tiling, d, V, K, N):
             assert np.array_equal(a[k], b[k]), k
 
 
+def test_tiled_head_is_a_copy_and_borrowed_head_is_read_in_place():
+    """After rpd_set_head the tiled layout no longer reads the caller's W (overwriting W leaves
+    the outputs unchanged); the borrowed layout reads it at every step (the same overwrite
+    changes them).  Unknown layouts are refused."""
+    case = small_case(1401, K=2, N=48, d=256, V=4100, w_std=0.08)
+    outs = {}
+    for layout in ("tiled", "borrowed"):
+        runner = DeviceRunner(case["W"], case["g"], 2, case["eps"], rule=case["rule"], layout=layout)
+        try:
+            before = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+            runner.W.copy_(torch.flip(runner.W, dims=[0]))  # the caller's buffer, rows reversed
+            after = runner.step(case["hidden"], case["mask"], case["tau"], case["budget"])
+            outs[layout] = (before, after)
+        finally:
+            runner.close()
+    b, a = outs["tiled"]
+    assert np.array_equal(b["layer_argmax"], a["layer_argmax"]) and np.array_equal(b["conf"], a["conf"])
+    b, a = outs["borrowed"]
+    assert not np.array_equal(b["layer_argmax"], a["layer_argmax"])
+    import paper_2609_36452_gb300 as rpd
+    ctx = rpd.Rpd(256, 4100, 2, 1e-6)
+    try:
+        with pytest.raises(rpd.RpdError) as e:
+            rpd._check(rpd.rpd_set_head_layout(ctx.handle, 7))
+        assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+    finally:
+        ctx.close()
+
+
 @pytest.mark.parametrize("tiling", ["pair", "rows_n"])
 @pytest.mark.parametrize("rows", [1, 64, 127, 128, 129, 257, 320, 383, 384, 385, 513, 769, 832,
                                   895, 896, 897, 1023, 1025])
