@@ -25,8 +25,9 @@ constexpr int kPairStageBytesB = kPairHalfRows * kTileK * 2;
 // "Rows on N" tiles: a pair multiplies 256 vocabulary entries (128 per CTA, the MMA's M side)
 // by a group of up to 512 projected rows (the N side, in steps of 32), so rows are padded to a
 // multiple of 32 instead of a multiple of 256.  Each CTA stages its 128 head rows (16 KB) and
-// half of the group's rows per K-step; the accumulator of a group of at most 256 rows is
-// double-buffered in TMEM, a larger group uses all 512 columns once.
+// half of the group's rows per K-step; the accumulators of groups of at most 256 rows are
+// double-buffered in TMEM, groups of 288-320 rows go round a ring of 32-column TMEM chunks, and
+// larger groups use columns [0, G) in turn.
 constexpr int kSwapMaxRows = 512;
 constexpr int kSwapRowStep = 32;  // N of the M = 256 MMA: a multiple of 32, at least 32
 constexpr int kSwapMaxStages = 12;
