@@ -19,6 +19,7 @@ from __future__ import annotations
 
 import argparse
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -451,6 +452,7 @@ def run_rpd(args):
         # layer projected and the projection chosen per step on the device.
         trajectory = trajectory_runs(case["W"], case["g"], ["all", "auto"], graph=True, warm=1,
                                      tiling=args.tiling)
+        trajectory["device_loop"] = device_loop_runs(case["W"], case["g"])
     emit(args, case, R, flops, bytes_, ms_step, steps_s, ktimes, clocks, e2e,
          st[0] if B == 1 else st, world, extra_bytes=extra_bytes, trajectory=trajectory)
     if world > 1:
@@ -688,6 +690,114 @@ def trajectory_runs(W, g, projections, graph=True, warm=1, tiling="auto"):
             "peaks": {"bf16_tflops": peaks["bf16_tflops"], "hbm_gbs": peaks["hbm_gbs"],
                       "source": peaks["source"]},
             **results}
+
+
+def device_loop_runs(W, g, repeats=3):
+    """The LLaDA decode trajectory (N=256, K=4) with the decoding loop on the device: a
+    stand-in for the backbone's forward pass - torch ops, captured as a CUDA graph, that rebuild
+    the hidden states from the canvas before every step (the trajectory's generator: the signal
+    of position p grows as the canvas left of p is committed; its noise is drawn once) - and the
+    step repeat inside one graph launch until at most 2% of the canvas is masked
+    (rpd_build_decode_loop).  Timed with CUDA events around one launch.  The same forward pass
+    and step, replayed from the host with a read of the masked count after every step, are
+    timed beside it: the difference is what returning to the host between steps costs."""
+    import paper_2609_36452_gb300 as rpd
+    import workloads as WL
+    dev = torch.device("cuda:0")
+    K, N = 4, 256
+    V, d = W.shape
+    gen = torch.Generator().manual_seed(4004)
+    targets = torch.randint(0, V, (N,), generator=gen)
+    flip = torch.randperm(N, generator=gen)[: N // 10]
+    alt = (targets[flip] + torch.randint(1, V, (flip.numel(),), generator=gen)) % V
+    wt = W[targets].float()
+    wt = wt / wt.norm(dim=1, keepdim=True)
+    wf = wt.clone()
+    wf[flip] = W[alt].float() / W[alt].float().norm(dim=1, keepdim=True)
+    dirs = torch.stack([wf if k == K - 2 else wt for k in range(K)]).to(dev)
+    noise = torch.randn(K, N, d, generator=gen).to(dev)
+    a = WL.layer_ramp(K).to(dev)
+    base_b = WL.u_profile(N, 0.3, 4.0).to(dev)
+    sigma = WL.DEFAULT_KAPPA * math.sqrt(d)
+    pos = torch.arange(N, device=dev)
+    denom = pos.clamp_min(1).float()
+    hidden = torch.empty(K, N, d, dtype=torch.bfloat16, device=dev)
+    mask = torch.ones(N, dtype=torch.uint8, device=dev)
+    commit = torch.zeros(N, dtype=torch.uint8, device=dev)
+    token = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    stats = torch.zeros(rpd.STATS_WORDS, dtype=torch.int32, device=dev)
+    steps = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def forward():
+        committed = (mask == 0).float()
+        before = torch.cumsum(committed, 0) - committed
+        f = torch.where(pos > 0, before / denom, torch.ones_like(before))
+        b = base_b + (4.0 - base_b).clamp_min(0) * f.pow(8)
+        hidden.copy_((a[:, None, None] * sigma * b[None, :, None] * dirs + noise).to(torch.bfloat16))
+
+    stream = torch.cuda.current_stream(dev)
+    ctx = rpd.Rpd(d, V, K, 1e-6)
+    ctx.set_stream(stream)
+    ctx.set_head(W.to(dev), g.to(dev))
+    ctx.set_profile("llada")
+    ctx.reserve(1, N)
+    try:
+        fwd_graph = torch.cuda.CUDAGraph(keep_graph=True)
+    except TypeError:
+        return {"unavailable": "this PyTorch cannot hand out a captured graph (keep_graph)"}
+    forward()
+    with torch.cuda.graph(fwd_graph):
+        forward()
+    fwd_graph.instantiate()
+    # the step alone, captured for the host-driven replay
+    step_graph = torch.cuda.CUDAGraph()
+    mask.fill_(1)
+    ctx.step(hidden, mask, 0.9, 1.0, commit, token, stats)
+    torch.cuda.synchronize(dev)
+    with torch.cuda.graph(step_graph):
+        ctx.set_stream(torch.cuda.current_stream(dev))
+        ctx.step(hidden, mask, 0.9, 1.0, commit, token, stats)
+    ctx.set_stream(stream)
+    loop = ctx.build_decode_loop(hidden, mask, 0.9, 1.0, commit, token, stats, steps,
+                                 stop_frac=0.02, max_steps=64, forward=fwd_graph)
+    dev_ms, host_ms = [], []
+    dev_steps = host_steps = 0
+    for _ in range(repeats + 1):
+        mask.fill_(1)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        loop.launch(stream)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        dev_ms.append(e0.elapsed_time(e1))
+        dev_steps = int(steps.item())
+        mask.fill_(1)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        n = 0
+        while True:
+            fwd_graph.replay()
+            step_graph.replay()
+            n += 1
+            st = rpd.stats_dict(stats.cpu())  # the host reads the step's result
+            if st["status"] != 0 or st["n_masked"] - st["n_committed"] <= int(0.02 * N) or n >= 64:
+                break
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        host_ms.append(e0.elapsed_time(e1))
+        host_steps = n
+    loop.close()
+    ctx.close()
+    dev_t, host_t = sorted(dev_ms[1:])[len(dev_ms[1:]) // 2], sorted(host_ms[1:])[len(host_ms[1:]) // 2]
+    return {"workload": "llada_trajectory_device_loop (N=256, K=4, d=4096, V=126464; forward "
+                        "stand-in rebuilds the hidden states from the canvas on the device)",
+            "steps": dev_steps, "total_ms": round(dev_t, 4), "steps_per_s": dev_steps / (dev_t / 1e3),
+            "host_loop": {"steps": host_steps, "total_ms": round(host_t, 4),
+                          "timing": "forward and step graph replays, host read of the step's "
+                                    "statistics after every step"},
+            "timing": f"median of {repeats} launches, CUDA events around one launch"}
 
 
 def run_trajectory(args):

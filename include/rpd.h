@@ -171,6 +171,36 @@ int rpd_set_projection(rpd_ctx *ctx, int mode);
 #define RPD_TILING_ROWS_N 2
 int rpd_set_head_tiling(rpd_ctx *ctx, int tiling);
 
+/* Decoding loop with device-side stopping.  The paper's decoder alternates the model's forward
+ * pass with the commit step until the canvas is complete (§3; App. A.6).  This builds a CUDA
+ * graph whose one launch repeats on the device, without returning to the host:
+ *   1. `forward`, a cudaGraph_t the caller built (for instance by stream capture): the
+ *      backbone's forward pass, which writes the next step's hidden states into `hidden` from
+ *      the canvas as it stands (NULL: the hidden states are not refreshed, for tests and
+ *      measurements);
+ *   2. one rpd_step(hidden, mask, N, tau, budget, out_commit, out_token, out_stats) on the
+ *      context, with its rule, projection and head tiling as they are at build time;
+ *   3. a stop test: the loop ends once at most floor(stop_frac * N) positions remain masked,
+ *      after max_steps steps, or when the step's status is not RPD_OK;
+ * and runs steps 1-3 at least once per launch.  steps (device int32) receives the number of
+ * steps run, out_stats the last step's statistics, out_commit and out_token the last step's
+ * commits (mask holds the canvas's remaining masked positions).  The graph is instantiated
+ * into *out_exec (a cudaGraphExec_t): launch it with rpd_decode_loop_launch (or
+ * cudaGraphLaunch) on any stream and free it with rpd_decode_loop_destroy; `forward` is copied
+ * into it and stays the caller's.  Scratch is reserved for one canvas of N positions while
+ * building.  hidden and mask are device memory (hidden 16-byte aligned).
+ * Requires 1 <= N <= 8192, 0 <= stop_frac <= 1, max_steps >= 1; a context holding a vocabulary
+ * slice is refused with RPD_ERR_UNSUPPORTED.  Errors from building the graph: RPD_ERR_CUDA. */
+int rpd_build_decode_loop(rpd_ctx *ctx, void *forward, const void *hidden, uint8_t *mask, int N,
+                          float tau, float budget, uint8_t *out_commit, int32_t *out_token,
+                          rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
+                          void **out_exec);
+/* Launch a decoding loop built by rpd_build_decode_loop on `stream` (a cudaStream_t, NULL =
+ * legacy default stream), asynchronously.  Free it with rpd_decode_loop_destroy (NULL is
+ * ignored) once no launch of it is in flight. */
+int rpd_decode_loop_launch(void *exec, void *stream);
+void rpd_decode_loop_destroy(void *exec);
+
 /* Diagnostics.  Every wait inside the step's kernels (mbarrier waits of the head kernels) is
  * bounded; when one runs out the kernel stops, drains what it has in flight, frees its
  * tensor memory and latches RPD_ERR_TIMEOUT in rpd_stats.status (the other outputs of that

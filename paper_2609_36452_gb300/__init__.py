@@ -18,6 +18,7 @@ __all__ = [
     "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_head_layout", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_set_vocab_shard",
     "rpd_step_shard_partials", "rpd_step_shard_finish", "rpd_profile_enable", "rpd_kernel_times",
+    "rpd_build_decode_loop", "rpd_decode_loop_launch", "rpd_decode_loop_destroy", "DecodeLoop",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
 
@@ -109,6 +110,10 @@ def _load():
         "rpd_set_vocab_shard": (i32, [vp, i32, i32]),
         "rpd_step_shard_partials": (i32, [vp, vp, vp, i32, vp]),
         "rpd_step_shard_finish": (i32, [vp, vp, i32, vp, i32, f32, f32, vp, vp, vp]),
+        "rpd_build_decode_loop": (i32, [vp, vp, vp, vp, i32, f32, f32, vp, vp, vp, f32, i32, vp,
+                                        ctypes.POINTER(vp)]),
+        "rpd_decode_loop_launch": (i32, [vp, vp]),
+        "rpd_decode_loop_destroy": (None, [vp]),
         "rpd_profile_enable": (i32, [vp, i32]),
         "rpd_kernel_times": (i32, [vp, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_int64), i32]),
@@ -134,6 +139,9 @@ rpd_reserve = lib.rpd_reserve
 rpd_set_debug = lib.rpd_set_debug
 rpd_set_projection = lib.rpd_set_projection
 rpd_set_head_tiling = lib.rpd_set_head_tiling
+rpd_build_decode_loop = lib.rpd_build_decode_loop
+rpd_decode_loop_launch = lib.rpd_decode_loop_launch
+rpd_decode_loop_destroy = lib.rpd_decode_loop_destroy
 rpd_set_head_layout = lib.rpd_set_head_layout
 rpd_set_wait_limit = lib.rpd_set_wait_limit
 rpd_inject_stall = lib.rpd_inject_stall
@@ -180,6 +188,30 @@ def _arg(t, name: str, dtype: str, numel: int = None, cuda: bool = True):
 _DEBUG_DTYPES = {"conf": "float32", "entropy": "float32", "persist": "int32", "drop": "float32",
                  "stability": "float32", "candidate": "uint8", "layer_argmax": "int32",
                  "layer_pmax": "float32"}
+
+
+class DecodeLoop:
+    """An instantiated decoding-loop graph (rpd_build_decode_loop): ``launch(stream)`` runs the
+    whole loop asynchronously on ``stream`` (a torch.cuda.Stream, or None for the current one)."""
+
+    def __init__(self, handle):
+        self.handle = handle
+
+    def launch(self, stream=None):
+        import torch
+        s = stream if stream is not None else torch.cuda.current_stream()
+        _check(rpd_decode_loop_launch(self.handle, ctypes.c_void_p(s.cuda_stream)))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            rpd_decode_loop_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 class Rpd:
@@ -282,6 +314,28 @@ class Rpd:
                 _arg(out_stats, "out_stats", "int32", STATS_WORDS))
         _check(rpd_step(self.handle, args[0], args[1], N, ctypes.c_float(tau),
                         ctypes.c_float(budget), *args[2:]))
+
+    def build_decode_loop(self, hidden, mask, tau, budget, out_commit, out_token, out_stats,
+                          steps, stop_frac=0.02, max_steps=64, forward=None):
+        """A CUDA graph that repeats [forward; step; stop test] on the device until at most
+        floor(stop_frac * N) positions remain masked (or max_steps steps, or an error status).
+        ``forward``: None, a torch.cuda.CUDAGraph built with keep_graph=True (the backbone's
+        forward pass writing ``hidden`` from the canvas), or a raw cudaGraph_t handle.
+        ``steps``: a CUDA int32 tensor of one element (steps run).  Returns a DecodeLoop."""
+        N = mask.numel()
+        fwd = None
+        if forward is not None:
+            fwd = forward.raw_cuda_graph() if hasattr(forward, "raw_cuda_graph") else int(forward)
+        exe = ctypes.c_void_p()
+        _check(rpd_build_decode_loop(
+            self.handle, fwd, _arg(hidden, "hidden", "bfloat16", self.K * N * self.d),
+            _arg(mask, "mask", "uint8", N), N, ctypes.c_float(tau), ctypes.c_float(budget),
+            _arg(out_commit, "out_commit", "uint8", N), _arg(out_token, "out_token", "int32", N),
+            _arg(out_stats, "out_stats", "int32", STATS_WORDS), ctypes.c_float(stop_frac),
+            int(max_steps), _arg(steps, "steps", "int32", 1), ctypes.byref(exe)))
+        loop = DecodeLoop(exe.value)
+        loop._keep = [hidden, mask, out_commit, out_token, out_stats, steps, forward, self]
+        return loop
 
     def step_batched(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):
         """B canvases: hidden [K][B][N][d], mask/out_commit/out_token [B][N], out_stats

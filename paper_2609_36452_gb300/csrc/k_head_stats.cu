@@ -945,7 +945,7 @@ cudaError_t launch_head(const HeadMaps &maps, const HeadParams &p, int grid, cud
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 2;
+    cfg.numAttrs = t_no_pdl ? 1 : 2;
     return cudaLaunchKernelEx(&cfg, k_head, maps, p);
 }
 

@@ -469,6 +469,28 @@ cudaError_t launch_merge_score(const MergeArgs &mg, int32_t *meta, const int32_t
     return launch_pdl(k_merge_score<8>, g, t, 0, s, mg, meta, sel_list, p);
 }
 
+namespace {
+// The stop test of the decoding loop: one thread counts the step and keeps the loop going
+// while more than floor(stop_frac * N) positions remain masked, fewer than max_steps steps
+// have run and the step succeeded.
+__global__ void k_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int N,
+                            float stop_frac, int max_steps, int32_t *steps) {
+    const int n = *steps + 1;
+    *steps = n;
+    const int remaining = stats->n_masked - stats->n_committed;
+    const int limit = static_cast<int>(floorf(stop_frac * static_cast<float>(N)));
+    const bool more = stats->status == RPD_OK && remaining > limit && n < max_steps;
+    cudaGraphSetConditional(handle, more ? 1u : 0u);
+}
+}  // namespace
+
+cudaError_t launch_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int N,
+                             float stop_frac, int max_steps, int32_t *steps, cudaStream_t s) {
+    // a plain launch: it must see the finished step's statistics
+    k_loop_test<<<1, 1, 0, s>>>(handle, stats, N, stop_frac, max_steps, steps);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_merge_shards(const ShardMergeParams &p, int grid, cudaStream_t s) {
     return launch_pdl(k_merge_shards, dim3(grid), dim3(kMergeThreads), 0, s, p);
 }

@@ -664,6 +664,125 @@ int rpd_step(rpd_ctx *c, const void *hidden, uint8_t *mask, int N, float tau, fl
     return run_step(c, hidden, mask, 1, N, &tau, &budget, out_commit, out_token, out_stats);
 }
 
+namespace {
+
+// One attempt at the decoding-loop graph (see rpd_build_decode_loop); `no_pdl` records the
+// step's launches without programmatic dependencies.
+int build_decode_loop_once(rpd_ctx *c, cudaGraph_t forward, const void *hidden, uint8_t *mask,
+                           int N, float tau, float budget, uint8_t *out_commit, int32_t *out_token,
+                           rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
+                           bool no_pdl, cudaGraphExec_t *out_exec) {
+    cudaStream_t cs = nullptr;
+    cudaGraph_t g = nullptr;
+    cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaGraphCreate(&g, 0);
+    cudaGraphConditionalHandle handle = 0;
+    // the condition is 1 at the start of every launch: the body runs at least once
+    if (e == cudaSuccess) e = cudaGraphConditionalHandleCreate(&handle, g, 1, cudaGraphCondAssignDefault);
+    // steps = 0, then while (condition) { forward; step; stop test }
+    cudaGraphNode_t zero = nullptr, loop = nullptr;
+    if (e == cudaSuccess) {
+        cudaMemsetParams ms = {};
+        ms.dst = steps;
+        ms.value = 0;
+        ms.elementSize = 4;
+        ms.width = 1;
+        ms.height = 1;
+        e = cudaGraphAddMemsetNode(&zero, g, nullptr, 0, &ms);
+    }
+    cudaGraph_t body = nullptr;
+    if (e == cudaSuccess) {
+        cudaGraphNodeParams cp = {};
+        cp.type = cudaGraphNodeTypeConditional;
+        cp.conditional.handle = handle;
+        cp.conditional.type = cudaGraphCondTypeWhile;
+        cp.conditional.size = 1;
+        e = cudaGraphAddNode(&loop, g, &zero, nullptr, 1, &cp);
+        if (e == cudaSuccess) body = cp.conditional.phGraph_out[0];
+    }
+    cudaGraphNode_t fwd = nullptr;
+    if (e == cudaSuccess && forward) e = cudaGraphAddChildGraphNode(&fwd, body, nullptr, 0, forward);
+    int rc = RPD_OK;
+    if (e == cudaSuccess) {
+        e = cudaStreamBeginCaptureToGraph(cs, body, fwd ? &fwd : nullptr, nullptr, fwd ? 1 : 0,
+                                          cudaStreamCaptureModeThreadLocal);
+        if (e == cudaSuccess) {
+            cudaStream_t saved = c->stream;
+            const bool saved_profile = c->profile;
+            c->stream = cs;
+            c->profile = false;
+            t_no_pdl = no_pdl;
+            rc = run_step(c, hidden, mask, 1, N, &tau, &budget, out_commit, out_token, out_stats);
+            cudaError_t el = rc == RPD_OK ? launch_loop_test(handle, out_stats, N, stop_frac, max_steps,
+                                                             steps, cs)
+                                          : cudaSuccess;
+            t_no_pdl = false;
+            c->stream = saved;
+            c->profile = saved_profile;
+            cudaGraph_t captured = nullptr;
+            e = cudaStreamEndCapture(cs, &captured);
+            if (e == cudaSuccess) e = el;
+        }
+    }
+    cudaGraphExec_t exec = nullptr;
+    if (rc == RPD_OK && e == cudaSuccess) e = cudaGraphInstantiate(&exec, g, 0);
+    if (g) cudaGraphDestroy(g);
+    if (cs) cudaStreamDestroy(cs);
+    if (rc != RPD_OK) return rc;
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return cuda_fail(e, "decoding-loop graph");
+    }
+    *out_exec = exec;
+    return RPD_OK;
+}
+
+}  // namespace
+
+int rpd_build_decode_loop(rpd_ctx *c, void *forward, const void *hidden, uint8_t *mask, int N,
+                          float tau, float budget, uint8_t *out_commit, int32_t *out_token,
+                          rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
+                          void **out_exec) {
+    if (!c || !out_exec || !steps || !hidden || !mask || !out_commit || !out_token || !out_stats)
+        return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    *out_exec = nullptr;
+    if (N < 1 || N > kMaxCanvas) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be in [1, %d]", kMaxCanvas);
+    if (!(stop_frac >= 0.f && stop_frac <= 1.f))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "stop_frac must be in [0, 1]");
+    if (max_steps < 1) return fail(RPD_ERR_INVALID_ARGUMENT, "max_steps must be >= 1");
+    if (c->V_total > 0) return fail(RPD_ERR_UNSUPPORTED, "a vocabulary slice has no decoding loop");
+    DeviceGuard dg(c->device);
+    if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
+    if (!pointer_usable(steps, c->device, false) || !pointer_usable(mask, c->device, false) ||
+        !pointer_usable(hidden, c->device, false))
+        return fail(RPD_ERR_INVALID_ARGUMENT, "hidden, mask and steps must be device memory");
+    int rc = check_call(c, tau, budget);
+    if (rc) return rc;
+    rc = ensure_scratch(c, 1, N);  // nothing may allocate while the step is recorded
+    if (rc) return rc;
+    cudaGraphExec_t exec = nullptr;
+    rc = build_decode_loop_once(c, static_cast<cudaGraph_t>(forward), hidden, mask, N, tau, budget,
+                                out_commit, out_token, out_stats, stop_frac, max_steps, steps, false,
+                                &exec);
+    if (rc == RPD_ERR_CUDA)  // a loop body may refuse programmatic dependencies: plain order
+        rc = build_decode_loop_once(c, static_cast<cudaGraph_t>(forward), hidden, mask, N, tau,
+                                    budget, out_commit, out_token, out_stats, stop_frac, max_steps,
+                                    steps, true, &exec);
+    if (rc) return rc;
+    *out_exec = exec;
+    return RPD_OK;
+}
+
+int rpd_decode_loop_launch(void *exec, void *stream) {
+    if (!exec) return fail(RPD_ERR_INVALID_ARGUMENT, "null graph");
+    cudaError_t e = cudaGraphLaunch(static_cast<cudaGraphExec_t>(exec), static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? RPD_OK : cuda_fail(e, "cudaGraphLaunch");
+}
+
+void rpd_decode_loop_destroy(void *exec) {
+    if (exec) cudaGraphExecDestroy(static_cast<cudaGraphExec_t>(exec));
+}
+
 int rpd_step_batched(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const float *tau,
                      const float *budget, uint8_t *out_commit, int32_t *out_token,
                      rpd_stats *out_stats) {

@@ -242,6 +242,11 @@ struct ScoreParams {
 // Launch with programmatic stream serialisation, so that the kernel's prologue overlaps the
 // tail of its predecessor in the stream (the kernel itself waits with griddepcontrol.wait
 // before it reads what the predecessor wrote).
+// Set on a host thread while it records launches that may not carry programmatic dependencies
+// (a graph body that refuses them): the launches are then plainly stream-ordered, and the
+// kernels' griddepcontrol instructions have nothing to wait for.
+inline thread_local bool t_no_pdl = false;
+
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
                        cudaStream_t s, Args &&...args) {
@@ -254,7 +259,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = t_no_pdl ? 0 : 1;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
 }
 
@@ -326,6 +331,9 @@ cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t
                          int grid, cudaStream_t s);
 cudaError_t launch_band(const BandParams &p, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
+// Stop test of the decoding loop: counts the step and sets the loop's condition (one thread).
+cudaError_t launch_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int N,
+                             float stop_frac, int max_steps, int32_t *steps, cudaStream_t s);
 cudaError_t launch_merge_shards(const ShardMergeParams &p, int grid, cudaStream_t s);
 // The step's last merge fused with the scoring of its canvas (one canvas of at most
 // kFuseScoreMaxN positions); the separate score launch is then skipped.
