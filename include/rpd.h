@@ -185,9 +185,9 @@ int rpd_set_head_tiling(rpd_ctx *ctx, int tiling);
  * and runs steps 1-3 at least once per launch.  steps (device int32) receives the number of
  * steps run, out_stats the last step's statistics, out_commit and out_token the last step's
  * commits (mask holds the canvas's remaining masked positions).  The graph is instantiated
- * into *out_exec (a cudaGraphExec_t): launch it with rpd_decode_loop_launch (or
- * cudaGraphLaunch) on any stream and free it with rpd_decode_loop_destroy; `forward` is copied
- * into it and stays the caller's.  Scratch is reserved for one canvas of N positions while
+ * into *out_exec (a cudaGraphExec_t owned by the context): launch it with
+ * rpd_decode_loop_launch on any stream and free it with rpd_decode_loop_destroy; `forward` is
+ * copied into it and stays the caller's.  Scratch is reserved for one canvas of N positions while
  * building.  hidden and mask are device memory (hidden 16-byte aligned).
  * Requires 1 <= N <= 8192, 0 <= stop_frac <= 1, max_steps >= 1; a context holding a vocabulary
  * slice is refused with RPD_ERR_UNSUPPORTED.  Errors from building the graph: RPD_ERR_CUDA. */
@@ -195,11 +195,16 @@ int rpd_build_decode_loop(rpd_ctx *ctx, void *forward, const void *hidden, uint8
                           float tau, float budget, uint8_t *out_commit, int32_t *out_token,
                           rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
                           void **out_exec);
-/* Launch a decoding loop built by rpd_build_decode_loop on `stream` (a cudaStream_t, NULL =
- * legacy default stream), asynchronously.  Free it with rpd_decode_loop_destroy (NULL is
- * ignored) once no launch of it is in flight. */
-int rpd_decode_loop_launch(void *exec, void *stream);
-void rpd_decode_loop_destroy(void *exec);
+/* Launch a decoding loop built by rpd_build_decode_loop on this context on `stream` (a
+ * cudaStream_t, NULL = legacy default stream), asynchronously.  The loop records the context's
+ * scratch and head: once either has been reallocated or replaced (a step on a larger canvas,
+ * rpd_reserve growing scratch, rpd_set_head), the launch is refused with
+ * RPD_ERR_INVALID_ARGUMENT and the loop must be rebuilt.  rpd_decode_loop_destroy frees a loop
+ * once no launch of it is in flight (NULL or unknown handles are ignored); rpd_destroy frees the
+ * context's remaining loops.  The debug buffers set before building (rpd_set_debug) must stay
+ * valid while the loop is used. */
+int rpd_decode_loop_launch(rpd_ctx *ctx, void *exec, void *stream);
+void rpd_decode_loop_destroy(rpd_ctx *ctx, void *exec);
 
 /* Diagnostics.  Every wait inside the step's kernels (mbarrier waits of the head kernels) is
  * bounded; when one runs out the kernel stops, drains what it has in flight, frees its

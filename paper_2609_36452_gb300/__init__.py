@@ -112,8 +112,8 @@ def _load():
         "rpd_step_shard_finish": (i32, [vp, vp, i32, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_build_decode_loop": (i32, [vp, vp, vp, vp, i32, f32, f32, vp, vp, vp, f32, i32, vp,
                                         ctypes.POINTER(vp)]),
-        "rpd_decode_loop_launch": (i32, [vp, vp]),
-        "rpd_decode_loop_destroy": (None, [vp]),
+        "rpd_decode_loop_launch": (i32, [vp, vp, vp]),
+        "rpd_decode_loop_destroy": (None, [vp, vp]),
         "rpd_profile_enable": (i32, [vp, i32]),
         "rpd_kernel_times": (i32, [vp, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_int64), i32]),
@@ -194,18 +194,18 @@ class DecodeLoop:
     """An instantiated decoding-loop graph (rpd_build_decode_loop): ``launch(stream)`` runs the
     whole loop asynchronously on ``stream`` (a torch.cuda.Stream, or None for the current one)."""
 
-    def __init__(self, handle):
-        self.handle = handle
+    def __init__(self, ctx, handle):
+        self.ctx, self.handle = ctx, handle
 
     def launch(self, stream=None):
         import torch
         s = stream if stream is not None else torch.cuda.current_stream()
-        _check(rpd_decode_loop_launch(self.handle, ctypes.c_void_p(s.cuda_stream)))
+        _check(rpd_decode_loop_launch(self.ctx.handle, self.handle, ctypes.c_void_p(s.cuda_stream)))
 
     def close(self):
-        if getattr(self, "handle", None):
-            rpd_decode_loop_destroy(self.handle)
-            self.handle = None
+        if getattr(self, "handle", None) and getattr(self.ctx, "handle", None):
+            rpd_decode_loop_destroy(self.ctx.handle, self.handle)
+        self.handle = None
 
     def __del__(self):
         try:
@@ -333,8 +333,8 @@ class Rpd:
             _arg(out_commit, "out_commit", "uint8", N), _arg(out_token, "out_token", "int32", N),
             _arg(out_stats, "out_stats", "int32", STATS_WORDS), ctypes.c_float(stop_frac),
             int(max_steps), _arg(steps, "steps", "int32", 1), ctypes.byref(exe)))
-        loop = DecodeLoop(exe.value)
-        loop._keep = [hidden, mask, out_commit, out_token, out_stats, steps, forward, self]
+        loop = DecodeLoop(self, exe.value)
+        loop._keep = [hidden, mask, out_commit, out_token, out_stats, steps, forward]
         return loop
 
     def step_batched(self, hidden, mask, tau, budget, out_commit, out_token, out_stats):

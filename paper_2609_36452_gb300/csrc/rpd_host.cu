@@ -138,6 +138,12 @@ struct rpd_ctx {
     // profiling
     bool profile = false;
     std::vector<cudaEvent_t> ev_pool;
+
+    // decoding loops built on this context, with the generation of the buffers they were
+    // recorded against; the generation moves whenever scratch is reallocated or the head
+    // replaced, and a loop recorded against an older one is refused at launch
+    uint64_t buffers_gen = 0;
+    std::vector<std::pair<cudaGraphExec_t, uint64_t>> loops;
     std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_rec;
     size_t ev_next = 0;
 
@@ -257,6 +263,7 @@ int ensure_scratch(rpd_ctx *c, int B, int N) {
         c->free_scratch();
         return cuda_fail(e, "cudaMemsetAsync(scratch)");
     }
+    ++c->buffers_gen;
     c->cap_bn = new_bn;
     c->cap_b = new_b;
     c->cap_rows = static_cast<int>(rows);
@@ -546,6 +553,7 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
     if (c->W_tiled) cudaFree(c->W_tiled);
     c->W_tiled = nullptr;
     c->W = nullptr;
+    ++c->buffers_gen;
     CUtensorMap m2;
     int rc;
     if (c->head_layout == RPD_HEAD_TILED && c->d % 64 == 0) {
@@ -572,6 +580,7 @@ int rpd_set_head(rpd_ctx *c, const void *W_head, const void *g_norm) {
         if (rc) return rc;
     }
     c->maps.w128 = m2;
+    ++c->buffers_gen;
     c->W = W_head;
     c->g = g_norm;
     return RPD_OK;
@@ -769,18 +778,35 @@ int rpd_build_decode_loop(rpd_ctx *c, void *forward, const void *hidden, uint8_t
                                     budget, out_commit, out_token, out_stats, stop_frac, max_steps,
                                     steps, true, &exec);
     if (rc) return rc;
+    c->loops.push_back({exec, c->buffers_gen});
     *out_exec = exec;
     return RPD_OK;
 }
 
-int rpd_decode_loop_launch(void *exec, void *stream) {
-    if (!exec) return fail(RPD_ERR_INVALID_ARGUMENT, "null graph");
-    cudaError_t e = cudaGraphLaunch(static_cast<cudaGraphExec_t>(exec), static_cast<cudaStream_t>(stream));
-    return e == cudaSuccess ? RPD_OK : cuda_fail(e, "cudaGraphLaunch");
+int rpd_decode_loop_launch(rpd_ctx *c, void *exec, void *stream) {
+    if (!c || !exec) return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
+    for (const auto &l : c->loops) {
+        if (l.first != static_cast<cudaGraphExec_t>(exec)) continue;
+        if (l.second != c->buffers_gen)
+            return fail(RPD_ERR_INVALID_ARGUMENT,
+                        "the context's scratch or head changed after the loop was built: rebuild it");
+        DeviceGuard dg(c->device);
+        if (dg.err != cudaSuccess) return cuda_fail(dg.err, "cudaSetDevice");
+        cudaError_t e = cudaGraphLaunch(l.first, static_cast<cudaStream_t>(stream));
+        return e == cudaSuccess ? RPD_OK : cuda_fail(e, "cudaGraphLaunch");
+    }
+    return fail(RPD_ERR_INVALID_ARGUMENT, "not a decoding loop of this context");
 }
 
-void rpd_decode_loop_destroy(void *exec) {
-    if (exec) cudaGraphExecDestroy(static_cast<cudaGraphExec_t>(exec));
+void rpd_decode_loop_destroy(rpd_ctx *c, void *exec) {
+    if (!c || !exec) return;
+    for (size_t i = 0; i < c->loops.size(); ++i) {
+        if (c->loops[i].first != static_cast<cudaGraphExec_t>(exec)) continue;
+        DeviceGuard dg(c->device);
+        cudaGraphExecDestroy(c->loops[i].first);
+        c->loops.erase(c->loops.begin() + static_cast<long>(i));
+        return;
+    }
 }
 
 int rpd_step_batched(rpd_ctx *c, const void *hidden, uint8_t *mask, int B, int N, const float *tau,
@@ -983,6 +1009,7 @@ void rpd_destroy(rpd_ctx *c) {
     if (!c) return;
     DeviceGuard dg(c->device);
     cudaStreamSynchronize(c->stream);
+    for (auto &l : c->loops) cudaGraphExecDestroy(l.first);
     c->free_scratch();
     if (c->W_tiled) cudaFree(c->W_tiled);
     if (c->stage) cudaFree(c->stage);

@@ -157,7 +157,9 @@ def test_decode_loop_refusals():
                                        out["stats"].data_ptr(), ctypes.c_float(0.0), 10,
                                        host_steps.data_ptr(), ctypes.byref(exe))
         assert rc == rpd.RPD_ERR_INVALID_ARGUMENT and not exe.value  # host memory for steps
-        assert rpd.rpd_decode_loop_launch(None, None) == rpd.RPD_ERR_INVALID_ARGUMENT
+        assert rpd.rpd_decode_loop_launch(None, None, None) == rpd.RPD_ERR_INVALID_ARGUMENT
+        assert rpd.rpd_decode_loop_launch(ctx.handle, ctypes.c_void_p(12345), None) == \
+            rpd.RPD_ERR_INVALID_ARGUMENT  # not a loop of this context
     finally:
         ctx.close()
     shard = rpd.Rpd(case["d"], 2048, case["K"], case["eps"])
@@ -170,3 +172,41 @@ def test_decode_loop_refusals():
         assert e.value.code == rpd.RPD_ERR_UNSUPPORTED
     finally:
         shard.close()
+
+
+def test_loop_is_refused_after_scratch_or_head_change():
+    """A loop records the context's scratch and head: after scratch grows, or the head is
+    replaced, launching it is refused (it would read freed memory); a rebuilt loop runs."""
+    case = small_case(2104, K=2, N=32, d=256, V=4100, w_std=0.08)
+    ctx = context(case)
+    try:
+        hidden = case["hidden"].to(DEV).contiguous()
+        mask = case["mask"].to(DEV).clone()
+        out = outputs(case["N"])
+        steps = torch.zeros(1, dtype=torch.int32, device=DEV)
+
+        def build():
+            return ctx.build_decode_loop(hidden, mask, case["tau"], case["budget"], out["commit"],
+                                         out["token"], out["stats"], steps, stop_frac=0.5,
+                                         max_steps=4)
+        loop = build()
+        loop.launch()
+        torch.cuda.synchronize(DEV)
+        assert int(steps.item()) >= 1
+        ctx.reserve(1, 4 * case["N"])  # scratch reallocated
+        with pytest.raises(rpd.RpdError) as e:
+            loop.launch()
+        assert e.value.code == rpd.RPD_ERR_INVALID_ARGUMENT
+        loop.close()
+        loop = build()
+        mask.copy_(case["mask"].to(DEV))
+        loop.launch()
+        torch.cuda.synchronize(DEV)
+        ctx.set_head(case["W"].to(DEV), case["g"].to(DEV))  # head replaced
+        with pytest.raises(rpd.RpdError):
+            loop.launch()
+        loop.close()
+        kept = build()  # freed by the context's destruction
+    finally:
+        ctx.close()
+    kept.close()  # after the context: a no-op
