@@ -195,7 +195,17 @@ int rpd_build_decode_loop(rpd_ctx *ctx, void *forward, const void *hidden, uint8
                           float tau, float budget, uint8_t *out_commit, int32_t *out_token,
                           rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
                           void **out_exec);
-/* Launch a decoding loop built by rpd_build_decode_loop on this context on `stream` (a
+/* The decoding loop over B canvases of N positions (the rpd_step_batched layout: hidden
+ * [K][B][N][d], mask / out_commit / out_token [B][N], out_stats [B]; tau[B] and budget[B] are
+ * host arrays read at build time).  The loop runs while some canvas has more than
+ * floor(stop_frac * N) positions masked, fewer than max_steps steps have run and every
+ * canvas's step succeeded.  Requires 1 <= B <= 128; otherwise as rpd_build_decode_loop. */
+int rpd_build_decode_loop_batched(rpd_ctx *ctx, void *forward, const void *hidden, uint8_t *mask,
+                                  int B, int N, const float *tau, const float *budget,
+                                  uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats,
+                                  float stop_frac, int max_steps, int32_t *steps, void **out_exec);
+
+/* Launch a decoding loop built by rpd_build_decode_loop(_batched) on this context on `stream` (a
  * cudaStream_t, NULL = legacy default stream), asynchronously.  The loop records the context's
  * scratch and head: once either has been reallocated or replaced (a step on a larger canvas,
  * rpd_reserve growing scratch, rpd_set_head), the launch is refused with

@@ -18,7 +18,7 @@ __all__ = [
     "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_head_layout", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_set_vocab_shard",
     "rpd_step_shard_partials", "rpd_step_shard_finish", "rpd_profile_enable", "rpd_kernel_times",
-    "rpd_build_decode_loop", "rpd_decode_loop_launch", "rpd_decode_loop_destroy", "DecodeLoop",
+    "rpd_build_decode_loop", "rpd_build_decode_loop_batched", "rpd_decode_loop_launch", "rpd_decode_loop_destroy", "DecodeLoop",
     "rpd_destroy", "rpd_last_error", "rpd_version", "Rpd", "RULE_PROFILES", "KERNEL_NAMES",
 ]
 
@@ -112,6 +112,8 @@ def _load():
         "rpd_step_shard_finish": (i32, [vp, vp, i32, vp, i32, f32, f32, vp, vp, vp]),
         "rpd_build_decode_loop": (i32, [vp, vp, vp, vp, i32, f32, f32, vp, vp, vp, f32, i32, vp,
                                         ctypes.POINTER(vp)]),
+        "rpd_build_decode_loop_batched": (i32, [vp, vp, vp, vp, i32, i32, vp, vp, vp, vp, vp, f32, i32,
+                                                vp, ctypes.POINTER(vp)]),
         "rpd_decode_loop_launch": (i32, [vp, vp, vp]),
         "rpd_decode_loop_destroy": (None, [vp, vp]),
         "rpd_profile_enable": (i32, [vp, i32]),
@@ -140,6 +142,7 @@ rpd_set_debug = lib.rpd_set_debug
 rpd_set_projection = lib.rpd_set_projection
 rpd_set_head_tiling = lib.rpd_set_head_tiling
 rpd_build_decode_loop = lib.rpd_build_decode_loop
+rpd_build_decode_loop_batched = lib.rpd_build_decode_loop_batched
 rpd_decode_loop_launch = lib.rpd_decode_loop_launch
 rpd_decode_loop_destroy = lib.rpd_decode_loop_destroy
 rpd_set_head_layout = lib.rpd_set_head_layout
@@ -332,6 +335,27 @@ class Rpd:
             _arg(mask, "mask", "uint8", N), N, ctypes.c_float(tau), ctypes.c_float(budget),
             _arg(out_commit, "out_commit", "uint8", N), _arg(out_token, "out_token", "int32", N),
             _arg(out_stats, "out_stats", "int32", STATS_WORDS), ctypes.c_float(stop_frac),
+            int(max_steps), _arg(steps, "steps", "int32", 1), ctypes.byref(exe)))
+        loop = DecodeLoop(self, exe.value)
+        loop._keep = [hidden, mask, out_commit, out_token, out_stats, steps, forward]
+        return loop
+
+    def build_decode_loop_batched(self, hidden, mask, tau, budget, out_commit, out_token,
+                                  out_stats, steps, stop_frac=0.02, max_steps=64, forward=None):
+        """build_decode_loop over B canvases: hidden [K][B][N][d], mask / out_commit / out_token
+        [B][N], out_stats [B][STATS_WORDS]; tau and budget are length-B host sequences."""
+        B, N = mask.shape
+        fwd = None
+        if forward is not None:
+            fwd = forward.raw_cuda_graph() if hasattr(forward, "raw_cuda_graph") else int(forward)
+        taus = (ctypes.c_float * B)(*[float(x) for x in tau])
+        budgets = (ctypes.c_float * B)(*[float(x) for x in budget])
+        exe = ctypes.c_void_p()
+        _check(rpd_build_decode_loop_batched(
+            self.handle, fwd, _arg(hidden, "hidden", "bfloat16", self.K * B * N * self.d),
+            _arg(mask, "mask", "uint8", B * N), B, N, taus, budgets,
+            _arg(out_commit, "out_commit", "uint8", B * N), _arg(out_token, "out_token", "int32", B * N),
+            _arg(out_stats, "out_stats", "int32", B * STATS_WORDS), ctypes.c_float(stop_frac),
             int(max_steps), _arg(steps, "steps", "int32", 1), ctypes.byref(exe)))
         loop = DecodeLoop(self, exe.value)
         loop._keep = [hidden, mask, out_commit, out_token, out_stats, steps, forward]

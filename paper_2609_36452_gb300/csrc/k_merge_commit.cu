@@ -471,23 +471,26 @@ cudaError_t launch_merge_score(const MergeArgs &mg, int32_t *meta, const int32_t
 
 namespace {
 // The stop test of the decoding loop: one thread counts the step and keeps the loop going
-// while more than floor(stop_frac * N) positions remain masked, fewer than max_steps steps
-// have run and the step succeeded.
-__global__ void k_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int N,
+// while some canvas has more than floor(stop_frac * N) positions masked, fewer than max_steps
+// steps have run and every canvas's step succeeded.
+__global__ void k_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int B, int N,
                             float stop_frac, int max_steps, int32_t *steps) {
     const int n = *steps + 1;
     *steps = n;
-    const int remaining = stats->n_masked - stats->n_committed;
     const int limit = static_cast<int>(floorf(stop_frac * static_cast<float>(N)));
-    const bool more = stats->status == RPD_OK && remaining > limit && n < max_steps;
-    cudaGraphSetConditional(handle, more ? 1u : 0u);
+    bool ok = true, open = false;
+    for (int b = 0; b < B; ++b) {
+        ok = ok && stats[b].status == RPD_OK;
+        open = open || stats[b].n_masked - stats[b].n_committed > limit;
+    }
+    cudaGraphSetConditional(handle, ok && open && n < max_steps ? 1u : 0u);
 }
 }  // namespace
 
-cudaError_t launch_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int N,
+cudaError_t launch_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int B, int N,
                              float stop_frac, int max_steps, int32_t *steps, cudaStream_t s) {
     // a plain launch: it must see the finished step's statistics
-    k_loop_test<<<1, 1, 0, s>>>(handle, stats, N, stop_frac, max_steps, steps);
+    k_loop_test<<<1, 1, 0, s>>>(handle, stats, B, N, stop_frac, max_steps, steps);
     return cudaGetLastError();
 }
 

@@ -678,9 +678,9 @@ namespace {
 // One attempt at the decoding-loop graph (see rpd_build_decode_loop); `no_pdl` records the
 // step's launches without programmatic dependencies.
 int build_decode_loop_once(rpd_ctx *c, cudaGraph_t forward, const void *hidden, uint8_t *mask,
-                           int N, float tau, float budget, uint8_t *out_commit, int32_t *out_token,
-                           rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
-                           bool no_pdl, cudaGraphExec_t *out_exec) {
+                           int B, int N, const float *tau, const float *budget, uint8_t *out_commit,
+                           int32_t *out_token, rpd_stats *out_stats, float stop_frac, int max_steps,
+                           int32_t *steps, bool no_pdl, cudaGraphExec_t *out_exec) {
     cudaStream_t cs = nullptr;
     cudaGraph_t g = nullptr;
     cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
@@ -721,9 +721,9 @@ int build_decode_loop_once(rpd_ctx *c, cudaGraph_t forward, const void *hidden, 
             c->stream = cs;
             c->profile = false;
             t_no_pdl = no_pdl;
-            rc = run_step(c, hidden, mask, 1, N, &tau, &budget, out_commit, out_token, out_stats);
-            cudaError_t el = rc == RPD_OK ? launch_loop_test(handle, out_stats, N, stop_frac, max_steps,
-                                                             steps, cs)
+            rc = run_step(c, hidden, mask, B, N, tau, budget, out_commit, out_token, out_stats);
+            cudaError_t el = rc == RPD_OK ? launch_loop_test(handle, out_stats, B, N, stop_frac,
+                                                             max_steps, steps, cs)
                                           : cudaSuccess;
             t_no_pdl = false;
             c->stream = saved;
@@ -748,13 +748,17 @@ int build_decode_loop_once(rpd_ctx *c, cudaGraph_t forward, const void *hidden, 
 
 }  // namespace
 
-int rpd_build_decode_loop(rpd_ctx *c, void *forward, const void *hidden, uint8_t *mask, int N,
-                          float tau, float budget, uint8_t *out_commit, int32_t *out_token,
-                          rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
-                          void **out_exec) {
-    if (!c || !out_exec || !steps || !hidden || !mask || !out_commit || !out_token || !out_stats)
+namespace {
+
+int build_decode_loop(rpd_ctx *c, void *forward, const void *hidden, uint8_t *mask, int B, int N,
+                      const float *tau, const float *budget, uint8_t *out_commit, int32_t *out_token,
+                      rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
+                      void **out_exec) {
+    if (!c || !out_exec || !steps || !hidden || !mask || !out_commit || !out_token || !out_stats ||
+        !tau || !budget)
         return fail(RPD_ERR_INVALID_ARGUMENT, "null argument");
     *out_exec = nullptr;
+    if (B < 1 || B > kMaxBatch) return fail(RPD_ERR_INVALID_ARGUMENT, "B must be in [1, %d]", kMaxBatch);
     if (N < 1 || N > kMaxCanvas) return fail(RPD_ERR_INVALID_ARGUMENT, "N must be in [1, %d]", kMaxCanvas);
     if (!(stop_frac >= 0.f && stop_frac <= 1.f))
         return fail(RPD_ERR_INVALID_ARGUMENT, "stop_frac must be in [0, 1]");
@@ -765,22 +769,42 @@ int rpd_build_decode_loop(rpd_ctx *c, void *forward, const void *hidden, uint8_t
     if (!pointer_usable(steps, c->device, false) || !pointer_usable(mask, c->device, false) ||
         !pointer_usable(hidden, c->device, false))
         return fail(RPD_ERR_INVALID_ARGUMENT, "hidden, mask and steps must be device memory");
-    int rc = check_call(c, tau, budget);
-    if (rc) return rc;
-    rc = ensure_scratch(c, 1, N);  // nothing may allocate while the step is recorded
+    for (int b = 0; b < B; ++b) {
+        int rc = check_call(c, tau[b], budget[b]);
+        if (rc) return rc;
+    }
+    int rc = ensure_scratch(c, B, N);  // nothing may allocate while the step is recorded
     if (rc) return rc;
     cudaGraphExec_t exec = nullptr;
-    rc = build_decode_loop_once(c, static_cast<cudaGraph_t>(forward), hidden, mask, N, tau, budget,
+    rc = build_decode_loop_once(c, static_cast<cudaGraph_t>(forward), hidden, mask, B, N, tau, budget,
                                 out_commit, out_token, out_stats, stop_frac, max_steps, steps, false,
                                 &exec);
     if (rc == RPD_ERR_CUDA)  // a loop body may refuse programmatic dependencies: plain order
-        rc = build_decode_loop_once(c, static_cast<cudaGraph_t>(forward), hidden, mask, N, tau,
+        rc = build_decode_loop_once(c, static_cast<cudaGraph_t>(forward), hidden, mask, B, N, tau,
                                     budget, out_commit, out_token, out_stats, stop_frac, max_steps,
                                     steps, true, &exec);
     if (rc) return rc;
     c->loops.push_back({exec, c->buffers_gen});
     *out_exec = exec;
     return RPD_OK;
+}
+
+}  // namespace
+
+int rpd_build_decode_loop(rpd_ctx *c, void *forward, const void *hidden, uint8_t *mask, int N,
+                          float tau, float budget, uint8_t *out_commit, int32_t *out_token,
+                          rpd_stats *out_stats, float stop_frac, int max_steps, int32_t *steps,
+                          void **out_exec) {
+    return build_decode_loop(c, forward, hidden, mask, 1, N, &tau, &budget, out_commit, out_token,
+                             out_stats, stop_frac, max_steps, steps, out_exec);
+}
+
+int rpd_build_decode_loop_batched(rpd_ctx *c, void *forward, const void *hidden, uint8_t *mask,
+                                  int B, int N, const float *tau, const float *budget,
+                                  uint8_t *out_commit, int32_t *out_token, rpd_stats *out_stats,
+                                  float stop_frac, int max_steps, int32_t *steps, void **out_exec) {
+    return build_decode_loop(c, forward, hidden, mask, B, N, tau, budget, out_commit, out_token,
+                             out_stats, stop_frac, max_steps, steps, out_exec);
 }
 
 int rpd_decode_loop_launch(rpd_ctx *c, void *exec, void *stream) {

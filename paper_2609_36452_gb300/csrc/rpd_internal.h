@@ -332,7 +332,7 @@ cudaError_t launch_merge(const MergeArgs &mg, const int32_t *meta, const int32_t
 cudaError_t launch_band(const BandParams &p, cudaStream_t s);
 cudaError_t launch_score_commit(const ScoreParams &p, cudaStream_t s);
 // Stop test of the decoding loop: counts the step and sets the loop's condition (one thread).
-cudaError_t launch_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int N,
+cudaError_t launch_loop_test(cudaGraphConditionalHandle handle, const rpd_stats *stats, int B, int N,
                              float stop_frac, int max_steps, int32_t *steps, cudaStream_t s);
 cudaError_t launch_merge_shards(const ShardMergeParams &p, int grid, cudaStream_t s);
 // The step's last merge fused with the scoring of its canvas (one canvas of at most

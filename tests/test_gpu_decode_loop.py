@@ -210,3 +210,54 @@ def test_loop_is_refused_after_scratch_or_head_change():
     finally:
         ctx.close()
     kept.close()  # after the context: a no-op
+
+
+def test_batched_device_loop_matches_host_loop():
+    """Three canvases of different masked fractions and thresholds: the loop runs until every
+    canvas is down to floor(stop_frac * N) masked positions; the host loop of rpd_step_batched
+    reaches the same state."""
+    import workloads as WL
+    B, N, K, d, V = 3, 48, 3, 256, 4100
+    W, g = WL.make_head(V, d, 2105, w_std=0.08)
+    b = WL.u_profile(N, 0.5, 3.0)
+    sigma = WL.calibrated_sigma(V, d, 0.08, b_max=float(b.max()))
+    hidden = torch.stack([WL.make_hidden(W, K, N, 3000 + i, b, sigma, flip_frac=0.1).hidden
+                          for i in range(B)], dim=1).to(DEV).contiguous()
+    mask0 = torch.stack([WL.uniform_fraction_mask(N, f, 40 + i)
+                         for i, f in enumerate((1.0, 0.6, 0.8))]).to(DEV)
+    taus, budgets = [0.9, 0.85, 0.95], [1.0, 2.0, 0.5]
+    ctx = rpd.Rpd(d, V, K, 1e-6)
+    ctx.set_stream(torch.cuda.current_stream(DEV))
+    ctx.set_head(W.to(DEV), g.to(DEV))
+    ctx.set_profile("llada")
+    ctx.reserve(B, N)
+
+    def outs():
+        return dict(commit=torch.zeros(B, N, dtype=torch.uint8, device=DEV),
+                    token=torch.full((B, N), -1, dtype=torch.int32, device=DEV),
+                    stats=torch.zeros(B, rpd.STATS_WORDS, dtype=torch.int32, device=DEV))
+    try:
+        stop_frac, limit = 0.1, int(np.floor(0.1 * N))
+        m_host, oh = mask0.clone(), outs()
+        n = 0
+        while True:
+            ctx.step_batched(hidden, m_host, taus, budgets, oh["commit"], oh["token"], oh["stats"])
+            n += 1
+            st = [rpd.stats_dict(oh["stats"][i].cpu()) for i in range(B)]
+            if any(x["status"] != 0 for x in st) or \
+                    all(x["n_masked"] - x["n_committed"] <= limit for x in st) or n >= 100:
+                break
+        m_dev, od = mask0.clone(), outs()
+        steps = torch.zeros(1, dtype=torch.int32, device=DEV)
+        loop = ctx.build_decode_loop_batched(hidden, m_dev, taus, budgets, od["commit"], od["token"],
+                                             od["stats"], steps, stop_frac=stop_frac, max_steps=100)
+        loop.launch()
+        torch.cuda.synchronize(DEV)
+        loop.close()
+        assert int(steps.item()) == n
+        assert torch.equal(m_host, m_dev)
+        assert torch.equal(oh["commit"], od["commit"]) and torch.equal(oh["token"], od["token"])
+        assert torch.equal(oh["stats"], od["stats"])
+        assert all(int(m_dev[i].sum()) <= limit for i in range(B))
+    finally:
+        ctx.close()
