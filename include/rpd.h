@@ -43,6 +43,8 @@ extern "C" {
 #define RPD_ERR_OUT_OF_MEMORY 4    /* scratch allocation failed */
 #define RPD_ERR_TIMEOUT 5          /* a kernel's bounded wait ran out (latched in rpd_stats.status) */
 #define RPD_ERR_UNSUPPORTED 6      /* shape outside what the kernels handle */
+#define RPD_ERR_CHECK 7            /* a device-side bounds check failed (only in a library built
+                                      with RPD_CHECKS; latched in rpd_stats.status) */
 
 typedef struct rpd_ctx rpd_ctx; /* opaque, owned by the library */
 

@@ -13,7 +13,7 @@ import os
 
 __all__ = [
     "RPD_OK", "RPD_ERR_INVALID_ARGUMENT", "RPD_ERR_NO_HEAD", "RPD_ERR_CUDA",
-    "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RpdRule", "RpdStats",
+    "RPD_ERR_OUT_OF_MEMORY", "RPD_ERR_TIMEOUT", "RPD_ERR_UNSUPPORTED", "RPD_ERR_CHECK", "RpdRule", "RpdStats",
     "RpdDebug", "RpdError", "lib", "lib_path", "rpd_create", "rpd_set_head", "rpd_set_rule",
     "rpd_get_rule", "rpd_set_stream", "rpd_reserve", "rpd_set_debug", "rpd_set_projection", "rpd_set_head_tiling", "rpd_set_head_layout", "rpd_set_wait_limit", "rpd_inject_stall", "rpd_step",
     "rpd_step_batched", "rpd_step_host", "rpd_step_noalloc", "rpd_set_vocab_shard",
@@ -29,6 +29,7 @@ RPD_ERR_CUDA = 3
 RPD_ERR_OUT_OF_MEMORY = 4
 RPD_ERR_TIMEOUT = 5
 RPD_ERR_UNSUPPORTED = 6
+RPD_ERR_CHECK = 7
 RPD_NUM_KERNELS = 4
 KERNEL_NAMES = ("gather_norm", "head_stats", "merge", "score_commit")
 
@@ -41,7 +42,9 @@ RULE_PROFILES = {
     "dream_block": (0.6, 2.5, 20.0, 6, 32, 32),
 }
 
-lib_path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librpd.so")
+# RPD_LIBRARY names another build of the library (the tests' checked build, librpd_checked.so)
+lib_path = os.environ.get("RPD_LIBRARY") or os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                                                          "librpd.so")
 
 
 class RpdRule(ctypes.Structure):

@@ -151,7 +151,9 @@ __global__ void __launch_bounds__(kNormThreads) k_gather_norm(NormParams p) {
         const int sr = r - kr * sel;
         const int k = layer0 + kr;
         const int q = p.sel_list ? p.sel_list[sr] : sr;
+        if (!rpd_check(q >= 0 && q < p.BN, p.meta + kMetaStatus)) continue;  // warp-uniform
         const int pos = p.pos_of_q[q];
+        if (!rpd_check(pos >= 0 && pos < p.BN, p.meta + kMetaStatus)) continue;
         const uint4 *__restrict__ src =
             reinterpret_cast<const uint4 *>(p.hidden + (static_cast<size_t>(k) * p.BN + pos) * p.d);
         uint4 *__restrict__ dst = reinterpret_cast<uint4 *>(p.u + static_cast<size_t>(r) * p.d);

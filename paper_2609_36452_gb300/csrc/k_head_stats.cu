@@ -411,7 +411,7 @@ __device__ __forceinline__ void head_pair(const CUtensorMap *tmU, const CUtensor
                 if (lane == 0) mbar_arrive_cluster(acc_empty0 + acc * static_cast<uint32_t>(sizeof(uint64_t)));
             }
             if (!ok) break;
-            if (valid) {
+            if (valid && rpd_check(g < p.max_splits, p.meta + kMetaStatus)) {
                 p.partials[static_cast<size_t>(r) * p.max_splits + g] =
                     make_float4(run_m, run_s, run_t, __int_as_float(run_a));
             }
@@ -822,7 +822,7 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
                     acc4 = merge_stat(acc4, stats[s4 * ng + rl]);
                     stats[s4 * ng + rl] = kEmpty;
                 }
-                if (r < rows)
+                if (r < rows && rpd_check(2 * g + static_cast<int>(rank) < p.max_splits, p.meta + kMetaStatus))
                     p.partials[static_cast<size_t>(r) * p.max_splits + 2 * g + static_cast<int>(rank)] = acc4;
             }
             if (!epi_sync(sm.epi, epi_phase, abort_flag, p.wait_limit_ns)) break;

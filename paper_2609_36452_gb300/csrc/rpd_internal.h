@@ -263,6 +263,18 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
 }
 
+// Bounds checks of the checked build (compiled with -DRPD_CHECKS): a failed check latches
+// RPD_ERR_CHECK in the step's status word (`status`, device memory) and the guarded access is
+// skipped; without RPD_CHECKS every check is `true` and compiles away.
+#ifdef RPD_CHECKS
+__device__ __forceinline__ bool rpd_check(bool ok, const int32_t *status) {
+    if (!ok) atomicCAS(const_cast<int32_t *>(status), RPD_OK, RPD_ERR_CHECK);
+    return ok;
+}
+#else
+__device__ __forceinline__ bool rpd_check(bool, const int32_t *) { return true; }
+#endif
+
 // Record the message returned by rpd_last_error() on this host thread.
 void set_last_error(const char *msg);
 

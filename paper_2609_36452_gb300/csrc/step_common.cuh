@@ -65,7 +65,9 @@ __device__ int merge_pass_rows(const MergeArgs &mg, const int32_t *meta, const i
     const int gid = threadIdx.x / gs, gl = threadIdx.x % gs;
     for (int base = cta_slot * groups; base < total; base += cta_slots * groups) {  // uniform trips
         const int idx = base + gid;
-        const bool valid = idx < total;
+        const bool valid = idx < total &&
+                           rpd_check(splits <= mg.max_splits && (idx / span) * sel + s_begin +
+                                     (idx - (idx / span) * span) < rows, meta + kMetaStatus);
         Stat acc{-INFINITY, 0.f, 0.f, 0x7fffffff};
         int kr = 0, s = 0;
         if (valid) {

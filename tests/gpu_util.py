@@ -63,6 +63,8 @@ class DeviceRunner:
             r["layer_argmax"] = out["layer_argmax"][:, b].cpu().numpy()
             r["layer_pmax"] = out["layer_pmax"][:, b].cpu().numpy()
             r["stats"] = self.rpd.stats_dict(out["stats"][b].cpu())
+            # a library built with RPD_CHECKS latches a failed device-side bounds check here
+            assert r["stats"]["status"] != self.rpd.RPD_ERR_CHECK, "device-side bounds check failed"
             r["new_mask"] = mask[b].cpu().numpy()
             res.append(r)
         return res
