@@ -41,11 +41,11 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h", "paper_2609_36452_gb300/csrc/head_plan.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "de25d1fb9a11e19b"): 1.0536e9,
-    ("llada_tail_70_masked", "de25d1fb9a11e19b"): 1.0556e9,
-    ("llada_tail_5_masked", "de25d1fb9a11e19b"): 1.0410e9,
-    ("dream_mid_decode", "de25d1fb9a11e19b"): 1.1047e9,
-    ("batched_serving", "de25d1fb9a11e19b"): 8.783e9,
+    ("llada_first_step", "37a9d90d79e3406a"): 1.0485e9,
+    ("llada_tail_70_masked", "37a9d90d79e3406a"): 1.0554e9,
+    ("llada_tail_5_masked", "37a9d90d79e3406a"): 1.0409e9,
+    ("dream_mid_decode", "37a9d90d79e3406a"): 1.1025e9,
+    ("batched_serving", "37a9d90d79e3406a"): 8.805e9,
 }
 
 # Nominal dense rates of GB300 (context only; the fractions use the measured peaks).
