@@ -21,11 +21,12 @@ import paper_2609_36452_gb300 as rpd  # noqa: E402
 DEV = torch.device("cuda:0")
 
 
-def context(case):
+def context(case, projection="all", profile=None):
     c = rpd.Rpd(case["d"], case["V"], case["K"], case["eps"])
     c.set_stream(torch.cuda.current_stream(DEV))
     c.set_head(case["W"].to(DEV), case["g"].to(DEV))
-    c.set_profile(case["rule"])
+    c.set_profile(profile or case["rule"])
+    c.set_projection(projection)
     c.reserve(1, case["N"])
     return c
 
@@ -76,12 +77,17 @@ def same_state(a, b, mask_a, mask_b):
     assert rpd.stats_dict(oa["stats"].cpu()) == rpd.stats_dict(ob["stats"].cpu())
 
 
-@pytest.mark.parametrize("stop_frac,max_steps", [(0.0, 200), (0.25, 200), (0.0, 3)])
-def test_device_loop_matches_host_loop_without_forward(stop_frac, max_steps):
+@pytest.mark.parametrize("stop_frac,max_steps,projection,profile", [
+    (0.0, 200, "all", None), (0.25, 200, "all", None), (0.0, 3, "all", None),
+    (0.0, 200, "lazy", None),            # k_band and a second projection pass inside the loop
+    (0.0, 200, "auto", None),
+    (0.0, 200, "all", "llada_block"),    # RPD-block: the active block's positions only
+])
+def test_device_loop_matches_host_loop_without_forward(stop_frac, max_steps, projection, profile):
     """Fixed hidden states: every step commits at least one position, so the loop ends by the
     masked fraction or by max_steps."""
     case = small_case(2101, K=3, N=64, d=256, V=4100, w_std=0.08)
-    ctx = context(case)
+    ctx = context(case, projection, profile)
     try:
         hidden = case["hidden"].to(DEV).contiguous()
         m_host = case["mask"].to(DEV).clone()
