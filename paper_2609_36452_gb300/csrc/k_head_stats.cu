@@ -304,63 +304,64 @@ __device__ __forceinline__ void head_pair(const CUtensorMap *tmU, const CUtensor
             }
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            if (rank == 0) {
-                // ------------------------------------------------ MMA issuer (even CTA only)
-                constexpr uint32_t idesc = idesc_bf16_f32(kPairTileM, kTileN);
-                int stage = 0;
-                uint32_t phase = 0;
-                uint32_t tile_iter = 0;
-                bool ok = true;
-                UnitCursor uc;
-                while (ok) {
-                    if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+        if (rank == 0) {
+            // -------------------------------------------- MMA issuer (even CTA only): the whole
+            // warp runs the loop, one elected lane issues (every branch below is warp-uniform)
+            constexpr uint32_t idesc = idesc_bf16_f32(kPairTileM, kTileN);
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t tile_iter = 0;
+            bool ok = true;
+            UnitCursor uc;
+            while (ok) {
+                if (!mbar_wait_bounded_warp(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+                    break;
+                const int u = unit_ring[uc.slot];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&unit_empty[uc.slot]);
+                uc.advance();
+                if (u < 0) break;
+                int m, g, n0, n1;
+                tw.unit(u, m, g, n0, n1);
+                for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
+                    const uint32_t acc = tile_iter & 1u;
+                    const uint32_t acc_phase = (tile_iter >> 1) & 1u;
+                    if (!mbar_wait_bounded_warp(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
+                                                p.wait_limit_ns)) {
+                        ok = false;
                         break;
-                    const int u = unit_ring[uc.slot];
-                    mbar_arrive(&unit_empty[uc.slot]);
-                    uc.advance();
-                    if (u < 0) break;
-                    int m, g, n0, n1;
-                    tw.unit(u, m, g, n0, n1);
-                    for (int n = n0; ok && n < n1; ++n, ++tile_iter) {
-                        const uint32_t acc = tile_iter & 1u;
-                        const uint32_t acc_phase = (tile_iter >> 1) & 1u;
-                        if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
-                                               p.wait_limit_ns)) {
+                    }
+                    tc_fence_after_sync();
+                    const uint32_t d_tmem = tmem_base + acc * kTileN;
+                    for (int kb = 0; kb < num_kb; ++kb) {
+                        if (!mbar_wait_bounded_warp(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after_sync();
-                        const uint32_t d_tmem = tmem_base + acc * kTileN;
-                        for (int kb = 0; kb < num_kb; ++kb) {
-                            if (!mbar_wait_bounded(&full[stage], phase, abort_flag, p.wait_limit_ns)) {
-                                ok = false;
-                                break;
-                            }
-                            tc_fence_after_sync();
-                            const uint32_t a0 = smem_u32(sm.ring + stage * kStageBytes);
-                            const uint32_t b0 = a0 + kPairStageBytesA;
+                        const uint32_t a0 = smem_u32(sm.ring + stage * kStageBytes);
+                        const uint32_t b0 = a0 + kPairStageBytesA;
 #pragma unroll
-                            for (int kk = 0; kk < kTileK / 16; ++kk) {
-                                umma_bf16_pair(d_tmem, smem_desc_sw128(a0 + kk * 32),
-                                               smem_desc_sw128(b0 + kk * 32), idesc,
-                                               (kb > 0 || kk > 0) ? 1u : 0u);
-                            }
-                            umma_commit_pair_multicast(&empty[stage], 0x3);
-                            if (++stage == kPairStages) {
-                                stage = 0;
-                                phase ^= 1u;
-                            }
+                        for (int kk = 0; kk < kTileK / 16; ++kk) {
+                            umma_bf16_pair_warp(d_tmem, smem_desc_sw128(a0 + kk * 32),
+                                                smem_desc_sw128(b0 + kk * 32), idesc,
+                                                (kb > 0 || kk > 0) ? 1u : 0u);
                         }
-                        if (!ok) break;
-                        umma_commit_pair_multicast(&acc_full[acc], 0x3);
+                        umma_commit_pair_multicast_warp(&empty[stage], 0x3);
+                        if (++stage == kPairStages) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
                     }
+                    if (!ok) break;
+                    umma_commit_pair_multicast_warp(&acc_full[acc], 0x3);
                 }
-                umma_commit_pair_multicast(sm.drain, 0x3);
             }
-            // Both CTAs: every MMA writing this CTA's TMEM has completed before it is freed.
-            mbar_wait_drain(sm.drain, 0, p.wait_limit_ns);
+            umma_commit_pair_multicast_warp(sm.drain, 0x3);
         }
+        // Both CTAs: every MMA writing this CTA's TMEM has completed before it is freed.
+        if (lane == 0) mbar_wait_drain(sm.drain, 0, p.wait_limit_ns);
+        __syncwarp();
     } else if (warp < 6) {
         // ---------------------------------------------------------- epilogue (both CTAs)
         const int sub = warp & 3;
@@ -468,9 +469,8 @@ __device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, volatil
 // four sub-partitions' statistics of each row are combined and each CTA writes one partial
 // per row (the merge sees 2 partials per split).
 // The K-steps of one rows-on-N tile issued as kSegs MMAs per 16-wide step (one per column
-// segment).  A separate loop per segment count keeps the issuing thread's loop free of
-// branches: with the segment tests inside the loop the single issuing thread measured 60 %
-// slower per tile.
+// segment), run by the whole issuing warp.  A separate loop per segment count keeps the loop
+// free of branches: with the segment tests inside it a tile measured 60 % slower.
 template <int kSegs>
 __device__ __forceinline__ bool swap_tile_mmas(const HeadSmem &sm, int num_kb, int stages,
                                                int stage_bytes, int &stage, uint32_t &phase,
@@ -479,22 +479,22 @@ __device__ __forceinline__ bool swap_tile_mmas(const HeadSmem &sm, int num_kb, i
                                                uint32_t bo2, volatile int *abort_flag,
                                                uint64_t limit) {
     for (int kb = 0; kb < num_kb; ++kb) {
-        if (!mbar_wait_bounded(&sm.full[stage], phase, abort_flag, limit)) return false;
+        if (!mbar_wait_bounded_warp(&sm.full[stage], phase, abort_flag, limit)) return false;
         tc_fence_after_sync();
         const uint32_t a0 = smem_u32(sm.ring + stage * stage_bytes);
         const uint32_t b0 = a0 + kSwapStageBytesA;
 #pragma unroll
         for (int kk = 0; kk < kTileK / 16; ++kk) {
             const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
-            umma_bf16_pair(d0, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + kk * 32), id0, accum);
+            umma_bf16_pair_warp(d0, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + kk * 32), id0, accum);
             if (kSegs > 1)
-                umma_bf16_pair(d1, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + bo1 + kk * 32),
-                               id1, accum);
+                umma_bf16_pair_warp(d1, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + bo1 + kk * 32),
+                                    id1, accum);
             if (kSegs > 2)
-                umma_bf16_pair(d2, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + bo2 + kk * 32),
-                               id2, accum);
+                umma_bf16_pair_warp(d2, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + bo2 + kk * 32),
+                                    id2, accum);
         }
-        umma_commit_pair_multicast(&sm.empty[stage], 0x3);
+        umma_commit_pair_multicast_warp(&sm.empty[stage], 0x3);
         if (++stage == stages) {
             stage = 0;
             phase ^= 1u;
@@ -656,72 +656,73 @@ __device__ __forceinline__ void head_swap(const CUtensorMap *tmUrows /* [kUMaps]
             }
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            if (rank == 0) {
-                // ------------------------------------------------ MMA issuer (even CTA only)
-                int stage = 0;
-                uint32_t phase = 0;
-                uint32_t tile_iter = 0;
-                bool ok = true;
-                UnitCursor uc;
-                while (ok) {
-                    if (!mbar_wait_bounded(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+        if (rank == 0) {
+            // -------------------------------------------- MMA issuer (even CTA only): the whole
+            // warp runs the loop, one elected lane issues (every branch below is warp-uniform)
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t tile_iter = 0;
+            bool ok = true;
+            UnitCursor uc;
+            while (ok) {
+                if (!mbar_wait_bounded_warp(&unit_full[uc.slot], uc.phase, abort_flag, p.wait_limit_ns))
+                    break;
+                const int u = unit_ring[uc.slot];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&unit_empty[uc.slot]);
+                uc.advance();
+                if (u < 0) break;
+                int m, g, v0, v1;
+                tw.unit(u, m, g, v0, v1);
+                for (int n = v0; ok && n < v1; ++n, ++tile_iter) {
+                    // tile t-2 read (its accumulator barrier is reused), or tile t-1 for tiles
+                    // that use all of TMEM ...
+                    const uint32_t acc = single ? 0u : (tile_iter & 1u);
+                    const uint32_t acc_phase = (single ? tile_iter : (tile_iter >> 1)) & 1u;
+                    if (!mbar_wait_bounded_warp(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
+                                                p.wait_limit_ns)) {
+                        ok = false;
                         break;
-                    const int u = unit_ring[uc.slot];
-                    mbar_arrive(&unit_empty[uc.slot]);
-                    uc.advance();
-                    if (u < 0) break;
-                    int m, g, v0, v1;
-                    tw.unit(u, m, g, v0, v1);
-                    for (int n = v0; ok && n < v1; ++n, ++tile_iter) {
-                        // tile t-2 read (its accumulator barrier is reused), or tile t-1 for tiles
-                        // that use all of TMEM ...
-                        const uint32_t acc = single ? 0u : (tile_iter & 1u);
-                        const uint32_t acc_phase = (single ? tile_iter : (tile_iter >> 1)) & 1u;
-                        if (!mbar_wait_bounded(&acc_empty[acc], acc_phase ^ 1u, abort_flag,
-                                               p.wait_limit_ns)) {
-                            ok = false;
-                            break;
-                        }
-                        // ... and, on the ring, the chunks of tile t-1 this tile overwrites
-                        const uint32_t a0 = tile_iter * nch;
-                        if (ring && tile_iter > 0) {
-                            for (uint32_t c = kChunks - nch; ok && c < nch; ++c) {
-                                const uint32_t a = a0 + c;  // previous use: a - 16, in tile t-1
-                                if (!mbar_wait_bounded(&chunk_free[a % kChunks], ((a / kChunks) & 1u) ^ 1u,
-                                                       abort_flag, p.wait_limit_ns))
-                                    ok = false;
-                            }
-                            if (!ok) break;
-                        }
-                        tc_fence_after_sync();
-                        const SwapSegs sg = swap_segments(static_cast<int>(ring ? a0 % kChunks : acc * 8u), ng);
-                        // (single: acc = 0, the tile starts at column 0)
-                        const uint32_t d0 = tmem_base + sg.col0, d1 = tmem_base + sg.col1,
-                                       d2 = tmem_base + sg.col2;
-                        const uint32_t id0 = idesc_bf16_f32(kPairTileM, sg.n0);
-                        const uint32_t id1 = idesc_bf16_f32(kPairTileM, sg.n1 > 0 ? sg.n1 : 32);
-                        const uint32_t id2 = idesc_bf16_f32(kPairTileM, sg.n2 > 0 ? sg.n2 : 32);
-                        // segment j's rows of u start at row (columns before it) / 2 of each CTA's half
-                        const uint32_t bo1 = static_cast<uint32_t>((sg.n0 / 2) * kTileK * 2);
-                        const uint32_t bo2 = static_cast<uint32_t>(((sg.n0 + sg.n1) / 2) * kTileK * 2);
-                        ok = sg.n2 > 0 ? swap_tile_mmas<3>(sm, num_kb, stages, stage_bytes, stage, phase, d0, d1,
-                                                           d2, id0, id1, id2, bo1, bo2, abort_flag,
-                                                           p.wait_limit_ns)
-                           : sg.n1 > 0 ? swap_tile_mmas<2>(sm, num_kb, stages, stage_bytes, stage, phase, d0,
-                                                           d1, d2, id0, id1, id2, bo1, bo2, abort_flag,
-                                                           p.wait_limit_ns)
-                                       : swap_tile_mmas<1>(sm, num_kb, stages, stage_bytes, stage, phase, d0,
-                                                           d1, d2, id0, id1, id2, bo1, bo2, abort_flag,
-                                                           p.wait_limit_ns);
-                        if (!ok) break;
-                        umma_commit_pair_multicast(&acc_full[acc], 0x3);
                     }
+                    // ... and, on the ring, the chunks of tile t-1 this tile overwrites
+                    const uint32_t a0 = tile_iter * nch;
+                    if (ring && tile_iter > 0) {
+                        for (uint32_t c = kChunks - nch; ok && c < nch; ++c) {
+                            const uint32_t a = a0 + c;  // previous use: a - 16, in tile t-1
+                            if (!mbar_wait_bounded_warp(&chunk_free[a % kChunks], ((a / kChunks) & 1u) ^ 1u,
+                                                        abort_flag, p.wait_limit_ns))
+                                ok = false;
+                        }
+                        if (!ok) break;
+                    }
+                    tc_fence_after_sync();
+                    const SwapSegs sg = swap_segments(static_cast<int>(ring ? a0 % kChunks : acc * 8u), ng);
+                    // (single: acc = 0, the tile starts at column 0)
+                    const uint32_t d0 = tmem_base + sg.col0, d1 = tmem_base + sg.col1,
+                                   d2 = tmem_base + sg.col2;
+                    const uint32_t id0 = idesc_bf16_f32(kPairTileM, sg.n0);
+                    const uint32_t id1 = idesc_bf16_f32(kPairTileM, sg.n1 > 0 ? sg.n1 : 32);
+                    const uint32_t id2 = idesc_bf16_f32(kPairTileM, sg.n2 > 0 ? sg.n2 : 32);
+                    // segment j's rows of u start at row (columns before it) / 2 of each CTA's half
+                    const uint32_t bo1 = static_cast<uint32_t>((sg.n0 / 2) * kTileK * 2);
+                    const uint32_t bo2 = static_cast<uint32_t>(((sg.n0 + sg.n1) / 2) * kTileK * 2);
+                    ok = sg.n2 > 0 ? swap_tile_mmas<3>(sm, num_kb, stages, stage_bytes, stage, phase, d0, d1,
+                                                       d2, id0, id1, id2, bo1, bo2, abort_flag,
+                                                       p.wait_limit_ns)
+                       : sg.n1 > 0 ? swap_tile_mmas<2>(sm, num_kb, stages, stage_bytes, stage, phase, d0,
+                                                       d1, d2, id0, id1, id2, bo1, bo2, abort_flag,
+                                                       p.wait_limit_ns)
+                                   : swap_tile_mmas<1>(sm, num_kb, stages, stage_bytes, stage, phase, d0,
+                                                       d1, d2, id0, id1, id2, bo1, bo2, abort_flag,
+                                                       p.wait_limit_ns);
+                    if (!ok) break;
+                    umma_commit_pair_multicast_warp(&acc_full[acc], 0x3);
                 }
-                umma_commit_pair_multicast(sm.drain, 0x3);
             }
-            mbar_wait_drain(sm.drain, 0, p.wait_limit_ns);
+            umma_commit_pair_multicast_warp(sm.drain, 0x3);
         }
+        if (lane == 0) mbar_wait_drain(sm.drain, 0, p.wait_limit_ns);
+        __syncwarp();
     } else {
         // ---------------------------------------------------------- epilogue (both CTAs)
         const int sub = warp & 3;                 // TMEM sub-partition (lanes 32*sub..+31)
