@@ -30,7 +30,11 @@ constexpr int kPairStageBytesB = kPairHalfRows * kTileK * 2;
 // larger groups use columns [0, G) in turn.
 constexpr int kSwapMaxRows = 512;
 constexpr int kSwapRowStep = 32;  // N of the M = 256 MMA: a multiple of 32, at least 32
-constexpr int kSwapMaxStages = 12;
+// At most 8 operand stages per CTA: small groups would fit 12, but with 12 the HBM-bound
+// head streamed 2 % slower (20 rows: 0.158 against 0.153 ms) - the extra copies in flight
+// bought nothing; 6 was slower again.  The barrier arrays are sized by this, so it must also
+// cover the pair tiling's stages.
+constexpr int kSwapMaxStages = 8;
 constexpr int kSwapStageBytesA = kPairHalfRows * kTileK * 2;
 
 constexpr int kSwapEpiWarps = 8;   // two per TMEM sub-partition, alternating its chunks
@@ -46,6 +50,7 @@ constexpr int kHeadBarrierBytes = 512;
 // The pair tiles' operand ring, or the rows-on-N ring, transpose blocks and statistics (the
 // ring takes what the other two leave): the 7-stage pair ring, 224 KB.
 constexpr int kHeadRegionBytes = 224 * 1024;
+static_assert(kPairStages <= kSwapMaxStages, "the stage barriers are shared by both tilings");
 static_assert(kPairStages * (kPairStageBytesA + kPairStageBytesB) <= kHeadRegionBytes,
               "the pair tiles' operand ring fits the region");
 static_assert(kHeadRegionBytes - kSwapXposeBytes - 4 * kSwapMaxRows * 16 >=
@@ -168,18 +173,18 @@ struct BandParams {
 // Costs of the tiling choice are in units of one 128-row x 256-entry tile's MMA work on one SM
 // at the nominal rate below (24.4 us).  The per-tile costs are measured ones (LLaDA head,
 // d = 4096, GB300, head time / tiles per pair, both tilings forced at 20 to 1024 rows):
-//   pair tile (256 rows x 256 entries per pair): 23.0 us, 0.943 units;
-//   rows-on-N tile (256 entries x a group of ng rows): 21.6 + 0.023 ng us (0.885 + 0.00094 ng
-//   units) for ng <= 256, whose accumulators are double-buffered, and 12.6 + 0.074 ng us
-//   (0.516 + 0.00303 ng units) for larger groups (288 rows: 34 us, 416: 43 us, 512: 50 us).
+//   pair tile (256 rows x 256 entries per pair): 22.3 us, 0.914 units;
+//   rows-on-N tile (256 entries x a group of ng rows): 20.5 + 0.025 ng us (0.840 + 0.00102 ng
+//   units) for ng <= 256, whose accumulators are double-buffered, and 4.9 + 0.0888 ng us
+//   (0.201 + 0.00364 ng units) for larger groups (288 rows: 30.5 us, 416: 42.8 us, 512: 50.4 us).
 // When streaming the head bounds a pass, pair tiles - half of whose staged bytes are rows of u -
-// stream it about 5 % slower than rows-on-N tiles (20 rows: 0.163 against 0.155 ms).
-constexpr float kPairTileCost = 0.943f;
-constexpr float kSwapTileBase = 0.885f;
-constexpr float kSwapTilePerRow = 0.00094f;
-constexpr float kSwapWideTileBase = 0.516f;
-constexpr float kSwapWideTilePerRow = 0.00303f;
-constexpr float kPairStreamFactor = 1.05f;
+// stream it about 4 % slower than rows-on-N tiles (20 rows: 0.159 against 0.153 ms).
+constexpr float kPairTileCost = 0.914f;
+constexpr float kSwapTileBase = 0.840f;
+constexpr float kSwapTilePerRow = 0.00102f;
+constexpr float kSwapWideTileBase = 0.201f;
+constexpr float kSwapWideTilePerRow = 0.00364f;
+constexpr float kPairStreamFactor = 1.04f;
 // Per-SM MMA rate of the unit tile and the sustained HBM read rate used by the tiling choice
 // (GB300 measurements; only their ratio matters).
 constexpr double kSingleTileFlopsPerSm = 1.1e13;
