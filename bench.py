@@ -41,11 +41,11 @@ UNIT = "commit-steps/s"
 HEAD_SOURCES = ("paper_2609_36452_gb300/csrc/k_head_stats.cu", "paper_2609_36452_gb300/csrc/ptx.cuh",
                 "paper_2609_36452_gb300/csrc/rpd_internal.h", "paper_2609_36452_gb300/csrc/head_plan.h")
 HEAD_TRAFFIC = {
-    ("llada_first_step", "831d6d52fa877d71"): 1.0519e9,
-    ("llada_tail_70_masked", "831d6d52fa877d71"): 1.0551e9,
-    ("llada_tail_5_masked", "831d6d52fa877d71"): 1.0404e9,
-    ("dream_mid_decode", "831d6d52fa877d71"): 1.1035e9,
-    ("batched_serving", "831d6d52fa877d71"): 8.8575e9,
+    ("llada_first_step", "38d1ebfe76e73880"): 1.0519e9,
+    ("llada_tail_70_masked", "38d1ebfe76e73880"): 1.0551e9,
+    ("llada_tail_5_masked", "38d1ebfe76e73880"): 1.0404e9,
+    ("dream_mid_decode", "38d1ebfe76e73880"): 1.1035e9,
+    ("batched_serving", "38d1ebfe76e73880"): 8.8575e9,
 }
 
 # Nominal dense rates of GB300 (context only; the fractions use the measured peaks).

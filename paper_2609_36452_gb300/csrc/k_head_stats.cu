@@ -21,7 +21,8 @@
 //                padded to a multiple of 32), so that a pass whose row count is not a multiple
 //                of 256 pads by at most 31 rows per group.
 // Roles: warp 0 TMA producer (one thread), warp 1 TMEM owner (512 columns) and MMA issuer
-// (one thread, even CTA), warps 2-9 epilogue (pair tiles use warps 2-5).  Every wait is
+// (the whole warp in the even CTA, one elected lane issuing), warps 2-9 epilogue (pair tiles
+// use warps 2-5).  Every wait is
 // bounded; a timeout latches RPD_ERR_TIMEOUT in the step's status word and the CTA drains and
 // exits.
 #include <atomic>
